@@ -1,0 +1,244 @@
+"""Reference restatement of the dynamic logic's table lookup —
+TEST INFRASTRUCTURE ONLY.
+
+The paper's dynamic logic inspects the pending independent GEMMs, predicts the
+concurrency degree (CD) to run, and rewrites each GEMM's kernel to the
+globally optimized kernel for that CD (Sec. 4.3, Sec. 4.4).  Here the
+prediction is a lookup table profiled offline; this module restates, in plain
+Python and independently of the product's C++ planner, how a schedule follows
+from the table:
+
+1. Bucket each GEMM by its sizes: key = (floor(log2 M), floor(log2 N),
+   floor(log2 K), output dtype).  The paper's predictor reads M, N and K among
+   its features (Sec. 4.3); a log2 bucket is this table's stand-in for them.
+2. Look the key up.  A key the table lacks takes the stored key nearest in
+   L1 distance over the three log2 sizes, a differing output dtype adding 16;
+   ties go to the smallest stored key.  (Nearest-neighbour reuse of profiled
+   GEMMs echoes the KNN tuning shortcut, Sec. 7.4.)
+3. The CD actually run is the minimum of the preferred CD and the number of
+   GEMMs available (Sec. 4.3).
+4. Two or more distinct keys (heterogeneous GEMMs, Sec. 6.6): the paper runs
+   the whole set at once only if every key prefers at least the set's size,
+   and otherwise runs homogeneous groups, each with its own CD.  Generalized
+   to any number of keys: one block per key, blocks in decreasing order of
+   total FLOPs (ties: smaller key first), merged greedily with the next block
+   while every key in the merged group still prefers at least the merged
+   size.  With two keys this is exactly the paper's rule.  A single-key group
+   runs at min(preferred CD, its size); a merged group runs all its members
+   at once.
+5. Inside a group GEMMs take stream slots round-robin (member j -> slot
+   j mod CD), so at most CD run at once; each GEMM runs the table's kernel for
+   the smallest CD class (1, 2, 4, 8, 16) not below the group's CD.
+
+Forced policies give the paper's comparison configurations through the same
+schedule type (Sec. 5.4): ``sequential`` (isolation-tuned kernels one after
+another), ``default`` (isolation-tuned kernels, all GEMMs at once on their own
+streams), ``go`` (GO-Kernels, all GEMMs at once) and ``force_cd`` (GO-Kernels
+at a fixed CD).
+
+Binary formats written out here, independently of the C++ code:
+
+LUT file (little-endian): 8-byte magic ``GOLDYLUT``, u32 version (1), u32
+entry count, u32 variant-id bound, u32 SM count, 8 reserved bytes; then
+16-byte entries ``u8 lm, u8 ln, u8 lk, u8 out_dtype, u8 pref_cd, u8 flags,
+u16 variant[5]`` sorted strictly by (lm, ln, lk, out_dtype).
+
+Schedule bytes (little-endian u32 words): ``GSCH`` magic, version (1),
+n_gemms, n_groups, max_streams, flags; per group: cd, size, members...; per
+GEMM: group, variant, slot.
+"""
+from __future__ import annotations
+
+import struct
+from dataclasses import dataclass
+from typing import List, Optional, Sequence, Tuple
+
+LUT_MAGIC = b"GOLDYLUT"
+CD_CLASSES = (1, 2, 4, 8, 16)
+MAX_GEMMS = 64
+MAX_STREAMS = 16
+
+# planning policies (low 4 bits of flags); the forced CD sits in bits 8..15
+POLICY_AUTO = 0
+POLICY_SEQUENTIAL = 1
+POLICY_DEFAULT = 2
+POLICY_GO = 3
+POLICY_FORCE_CD = 4
+
+DTYPE_BF16 = 0
+DTYPE_F32 = 1
+
+
+class LutError(ValueError):
+    pass
+
+
+class PlanError(ValueError):
+    pass
+
+
+@dataclass(frozen=True)
+class Entry:
+    key: Tuple[int, int, int, int]
+    pref_cd: int
+    variants: Tuple[int, int, int, int, int]
+
+
+def parse_lut(data: bytes) -> Tuple[List[Entry], int]:
+    """Entries and the variant-id bound of a LUT file; raises LutError on any
+    malformed field."""
+    if len(data) < 32 or data[:8] != LUT_MAGIC:
+        raise LutError("bad magic")
+    version, n, n_variants, _sm = struct.unpack_from("<IIII", data, 8)
+    if version != 1:
+        raise LutError("bad version")
+    if len(data) != 32 + 16 * n:
+        raise LutError("bad size")
+    entries: List[Entry] = []
+    prev = None
+    for e in range(n):
+        lm, ln, lk, out, pref, _flags = struct.unpack_from("<6B", data, 32 + 16 * e)
+        vs = struct.unpack_from("<5H", data, 32 + 16 * e + 6)
+        key = (lm, ln, lk, out)
+        if prev is not None and key <= prev:
+            raise LutError("entries not strictly sorted")
+        if out not in (DTYPE_BF16, DTYPE_F32):
+            raise LutError("bad dtype")
+        if pref not in CD_CLASSES:
+            raise LutError("bad preferred cd")
+        if any(v >= n_variants for v in vs):
+            raise LutError("variant out of range")
+        prev = key
+        entries.append(Entry(key, pref, tuple(vs)))
+    if not entries:
+        raise LutError("empty table")
+    return entries, n_variants
+
+
+def write_lut(entries: Sequence[Entry], n_variants: int, sm_count: int = 0) -> bytes:
+    out = bytearray(LUT_MAGIC)
+    out += struct.pack("<IIIIII", 1, len(entries), n_variants, sm_count, 0, 0)
+    for e in sorted(entries, key=lambda x: x.key):
+        out += struct.pack("<6B", *e.key, e.pref_cd, 0)
+        out += struct.pack("<5H", *e.variants)
+    return bytes(out)
+
+
+def floor_log2(x: int) -> int:
+    """floor(log2 x) for x >= 1, and 0 for x == 0, clamped to a byte."""
+    if x <= 0:
+        return 0
+    return min(x.bit_length() - 1, 255)
+
+
+def bucket_key(M: int, N: int, K: int, out_dtype: int) -> Tuple[int, int, int, int]:
+    return (floor_log2(M), floor_log2(N), floor_log2(K), out_dtype)
+
+
+def lookup(entries: Sequence[Entry], key) -> Entry:
+    best = None
+    best_d = None
+    for e in entries:                       # entries are in increasing key order
+        d = (abs(e.key[0] - key[0]) + abs(e.key[1] - key[1]) + abs(e.key[2] - key[2])
+             + (16 if e.key[3] != key[3] else 0))
+        if best_d is None or d < best_d:    # strict: earlier (smaller) key wins ties
+            best, best_d = e, d
+    return best
+
+
+def cd_class_index(cd: int) -> int:
+    for idx, c in enumerate(CD_CLASSES):
+        if cd <= c:
+            return idx
+    return len(CD_CLASSES) - 1
+
+
+@dataclass(frozen=True)
+class Desc:
+    M: int
+    N: int
+    K: int
+    out_dtype: int
+
+
+def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
+    """Schedule as (groups, per_gemm, max_streams, flags): groups is a list of
+    (cd, members); per_gemm[i] = (group, variant, slot)."""
+    entries, _ = parse_lut(lut_bytes)
+    n = len(descs)
+    if n < 1 or n > MAX_GEMMS:
+        raise PlanError("bad count")
+    policy = flags & 0xF
+    forced = (flags >> 8) & 0xFF
+    if policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
+        raise PlanError("bad flags")
+    keys = [bucket_key(d.M, d.N, d.K, d.out_dtype) for d in descs]
+    ents = [lookup(entries, k) for k in keys]
+
+    def one_group(cd: int, cls_cd: Optional[int]):
+        cd = max(1, min(cd, n, MAX_STREAMS))
+        ci = cd_class_index(cd if cls_cd is None else cls_cd)
+        members = list(range(n))
+        return [(cd, members, [ents[i].variants[ci] for i in members])]
+
+    if policy == POLICY_SEQUENTIAL:
+        groups = one_group(1, 1)
+    elif policy == POLICY_DEFAULT:
+        groups = one_group(n, 1)
+    elif policy == POLICY_GO:
+        groups = one_group(n, None)
+    elif policy == POLICY_FORCE_CD:
+        groups = one_group(forced, None)
+    else:
+        blocks = []
+        for k in sorted(set(keys)):
+            members = [i for i in range(n) if keys[i] == k]
+            flops = sum(2 * descs[i].M * descs[i].N * descs[i].K for i in members)
+            blocks.append((-flops, k, members, ents[members[0]].pref_cd))
+        blocks.sort(key=lambda b: (b[0], b[1]))
+        merged = []                         # each: (members, min pref, n keys)
+        for _, _, members, pref in blocks:
+            if merged:
+                cur_members, cur_pref, cur_keys = merged[-1]
+                size = len(cur_members) + len(members)
+                if min(cur_pref, pref) >= size:
+                    merged[-1] = (cur_members + members, min(cur_pref, pref), cur_keys + 1)
+                    continue
+            merged.append((list(members), pref, 1))
+        groups = []
+        for members, pref, n_keys in merged:
+            cd = len(members) if n_keys > 1 else min(pref, len(members))
+            cd = max(1, min(cd, MAX_STREAMS))
+            ci = cd_class_index(cd)
+            groups.append((cd, members, [ents[i].variants[ci] for i in members]))
+
+    per_gemm = [None] * n
+    for g, (cd, members, variants) in enumerate(groups):
+        for j, (i, v) in enumerate(zip(members, variants)):
+            per_gemm[i] = (g, v, j % cd)
+    max_streams = max(cd for cd, _, _ in groups)
+    return [(cd, members) for cd, members, _ in groups], per_gemm, max_streams, flags
+
+
+def serialize(schedule) -> bytes:
+    groups, per_gemm, max_streams, flags = schedule
+    words = [0x48435347, 1, len(per_gemm), len(groups), max_streams, flags & 0xFFFFFFFF]
+    for cd, members in groups:
+        words += [cd, len(members)] + list(members)
+    for g, v, s in per_gemm:
+        words += [g, v, s]
+    return struct.pack("<%dI" % len(words), *words)
+
+
+def preferred_cd(speedup: dict, gain: float = 0.05, near: float = 0.01) -> int:
+    """Preferred CD from measured speedups over serial execution (Sec. 4.3:
+    the CD with the most speedup; Sec. 5.4: sequential unless some CD gains at
+    least 5%).  Among CDs whose speedup is within ``near`` (relative) of the
+    best, the smallest wins.  ``speedup[1]`` is 1 by definition."""
+    cands = {cd: s for cd, s in speedup.items() if cd in CD_CLASSES and cd != 1}
+    if not cands:
+        return 1
+    best = max(cands.values())
+    if best < 1.0 + gain:
+        return 1
+    return min(cd for cd, s in cands.items() if s >= best * (1.0 - near))

@@ -1,0 +1,182 @@
+"""Seeded synthetic GEMM sets (inputs only; no GEMM arithmetic in here).
+
+This module is the one place both the product path and the CPU oracle get
+their inputs from: it draws bf16 matrices from a seeded ``torch.Generator``
+on the CPU and hands them out as tensors and as raw uint16 bit patterns, so
+both sides read identical bits.  It imports nothing else from the package.
+
+The sets stand in for the paper's GEMMs from low-batch RNNs, Transformers and
+tensor-sliced layers (Sec. 5.2, Table "apps"); the paper's own list of 410 /
+1072 GEMM sizes is not available, so these shapes follow the workload
+families it describes:
+
+* ``pair_256``    — 2 x (M=256, N=256, K=512), U[-1, 1], seed 0, fp32 out.
+* ``ffn_slices``  — tensor-sliced Transformer FFN at low batch:
+                    4 x (M=128 tokens, N=1024, K=4096), N(0, 0.02), seed 1,
+                    bf16 out.
+* ``lstm_gates``  — LSTM gate GEMMs at small batch: 8 x (M=32, N=4096,
+                    K=1024), U[-0.1, 0.1], seed 2, fp32 out.
+* ``hetero_pair`` — two co-running models: 3 x (512, 1024, 1024) plus
+                    1 x (2048, 8192, 2048), N(0, 1/sqrt(K)), seed 3, fp32 out.
+* ``sweep``       — 64 sets of 2-16 GEMMs, M log-uniform in [16, 4096],
+                    N and K log-uniform in [256, 8192] rounded to multiples of
+                    64, U[-1, 1], fp32 out; set j uses seed 1000 + j.
+
+Drawing order (fixed, so a set is reproducible from its seed): for GEMM i in
+order, A_i (M x K) then B_i (K x N), each as fp32 values rounded to bf16
+(round to nearest even).  ``uniform[a, b]`` is ``a + (b - a) * rand``;
+``normal(0, s)`` is ``s * randn``.  For the sweep, the set's size and all
+shapes are drawn first from the same generator, then the values.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+from typing import List, Optional, Tuple
+
+import numpy as np
+import torch
+
+DTYPE_BF16 = 0
+DTYPE_F32 = 1
+
+
+@dataclass(frozen=True)
+class GemmSpec:
+    M: int
+    N: int
+    K: int
+    out_dtype: int              # DTYPE_BF16 or DTYPE_F32
+    dist: str                   # "uniform" or "normal"
+    scale: float                # half-width for uniform, std-dev for normal
+
+    @property
+    def flops(self) -> int:
+        return 2 * self.M * self.N * self.K
+
+    @property
+    def bytes(self) -> int:
+        """Algorithmic bytes: A and B read once, C written once."""
+        out = 2 if self.out_dtype == DTYPE_BF16 else 4
+        return 2 * self.M * self.K + 2 * self.K * self.N + out * self.M * self.N
+
+
+@dataclass
+class GemmSet:
+    name: str
+    seed: int
+    specs: List[GemmSpec]
+    a: List[torch.Tensor] = field(default_factory=list)   # bf16, CPU, M x K
+    b: List[torch.Tensor] = field(default_factory=list)   # bf16, CPU, K x N
+
+    @property
+    def flops(self) -> int:
+        return sum(s.flops for s in self.specs)
+
+    @property
+    def bytes(self) -> int:
+        return sum(s.bytes for s in self.specs)
+
+    def a_bits(self, i: int) -> np.ndarray:
+        return bits_of(self.a[i])
+
+    def b_bits(self, i: int) -> np.ndarray:
+        return bits_of(self.b[i])
+
+
+def bits_of(t: torch.Tensor) -> np.ndarray:
+    """Raw uint16 bit patterns of a bf16 CPU tensor (no copy of values)."""
+    assert t.dtype == torch.bfloat16
+    return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def _draw(gen: torch.Generator, rows: int, cols: int, dist: str, scale: float) -> torch.Tensor:
+    if dist == "uniform":
+        x = torch.rand((rows, cols), generator=gen, dtype=torch.float32)
+        x = -scale + (2.0 * scale) * x
+    elif dist == "normal":
+        x = scale * torch.randn((rows, cols), generator=gen, dtype=torch.float32)
+    else:
+        raise ValueError(dist)
+    return x.to(torch.bfloat16)
+
+
+def materialize(name: str, seed: int, specs: List[GemmSpec],
+                gen: Optional[torch.Generator] = None) -> GemmSet:
+    if gen is None:
+        gen = torch.Generator(device="cpu")
+        gen.manual_seed(seed)
+    s = GemmSet(name, seed, list(specs))
+    for sp in specs:
+        s.a.append(_draw(gen, sp.M, sp.K, sp.dist, sp.scale))
+        s.b.append(_draw(gen, sp.K, sp.N, sp.dist, sp.scale))
+    return s
+
+
+def config_specs(name: str) -> Tuple[int, List[GemmSpec]]:
+    """(seed, GEMM specs) of a named fixed configuration."""
+    if name == "pair_256":
+        return 0, [GemmSpec(256, 256, 512, DTYPE_F32, "uniform", 1.0)] * 2
+    if name == "ffn_slices":
+        return 1, [GemmSpec(128, 1024, 4096, DTYPE_BF16, "normal", 0.02)] * 4
+    if name == "lstm_gates":
+        return 2, [GemmSpec(32, 4096, 1024, DTYPE_F32, "uniform", 0.1)] * 8
+    if name == "hetero_pair":
+        small = GemmSpec(512, 1024, 1024, DTYPE_F32, "normal", 1.0 / math.sqrt(1024))
+        big = GemmSpec(2048, 8192, 2048, DTYPE_F32, "normal", 1.0 / math.sqrt(2048))
+        return 3, [small, small, small, big]
+    raise KeyError(name)
+
+
+FIXED_CONFIGS = ("pair_256", "ffn_slices", "lstm_gates", "hetero_pair")
+SWEEP_SETS = 64
+
+
+def make_config(name: str) -> GemmSet:
+    seed, specs = config_specs(name)
+    return materialize(name, seed, specs)
+
+
+def _log_uniform(gen: torch.Generator, lo: float, hi: float) -> float:
+    u = float(torch.rand((1,), generator=gen, dtype=torch.float64)[0])
+    return math.exp(math.log(lo) + u * (math.log(hi) - math.log(lo)))
+
+
+def sweep_specs(j: int) -> Tuple[int, List[GemmSpec], torch.Generator]:
+    """Shapes of sweep set j (0 <= j < 64) and the generator positioned for
+    drawing its values."""
+    seed = 1000 + j
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed)
+    n = 2 + int(torch.randint(0, 15, (1,), generator=gen)[0])      # 2..16
+    specs = []
+    for _ in range(n):
+        M = int(round(_log_uniform(gen, 16, 4096)))
+        M = min(max(M, 16), 4096)
+        N = 64 * int(round(_log_uniform(gen, 256, 8192) / 64))
+        N = min(max(N, 256), 8192)
+        K = 64 * int(round(_log_uniform(gen, 256, 8192) / 64))
+        K = min(max(K, 256), 8192)
+        specs.append(GemmSpec(M, N, K, DTYPE_F32, "uniform", 1.0))
+    return seed, specs, gen
+
+
+def make_sweep_set(j: int) -> GemmSet:
+    seed, specs, gen = sweep_specs(j)
+    return materialize(f"sweep_{j:02d}", seed, specs, gen)
+
+
+def random_matrix(rows: int, cols: int, seed: int, dist: str = "uniform",
+                  scale: float = 1.0) -> torch.Tensor:
+    """One seeded bf16 matrix (used for edge-case tests of odd shapes)."""
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed)
+    return _draw(gen, rows, cols, dist, scale)
+
+
+def integer_matrix(rows: int, cols: int, seed: int, lo: int = -8, hi: int = 8) -> torch.Tensor:
+    """Seeded bf16 matrix of small integers in [lo, hi] (exact in bf16)."""
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed)
+    x = torch.randint(lo, hi + 1, (rows, cols), generator=gen, dtype=torch.int32)
+    return x.to(torch.float32).to(torch.bfloat16)
