@@ -1,0 +1,223 @@
+/*
+ * goldy.h — C ABI of the concurrent-GEMM library (GO-Kernels + dynamic logic)
+ * for one GB300 (sm_103a).
+ *
+ * The paper's problem (Sec. 4.1, Sec. 4.4): a set of independent GEMMs is
+ * queued at once; the system picks how many run concurrently (the
+ * concurrency degree, CD) and, for each GEMM, a kernel tuned for the
+ * resources it will share at that CD (a "GO-Kernel"), then launches them.
+ * This header splits that into
+ *
+ *   goldy_plan()  host only, integer work, no CUDA call: GEMM descriptors +
+ *                 lookup table -> schedule (groups run one after another; in
+ *                 a group, CD streams; per GEMM a kernel variant and a stream
+ *                 slot).  The dynamic logic of Sec. 4.3 / Sec. 4.4.
+ *   goldy_run()   asynchronous launch of a schedule on caller-owned streams
+ *                 and caller-owned device buffers.  No allocation, no
+ *                 synchronisation.  The GO-Kernels themselves (Sec. 4.2).
+ *
+ * Conventions for every entry point:
+ *   - Return a goldy_status; nothing is thrown across the ABI.  On error the
+ *     thread-local text of goldy_last_error() says why.
+ *   - Pointers the caller passes stay owned by the caller.  Objects the
+ *     library returns (goldy_lut, goldy_schedule, goldy_graph) are owned by
+ *     the library and released with the matching *_free function.
+ *   - Device pointers are plain CUDA device addresses on the current device;
+ *     streams are cudaStream_t values passed as void*.
+ *
+ * Matrix layout (Sec. 2.1.2; transposes T1 = T2 = 0 in the K x N sense):
+ *   A: M x K, row-major, element (i, k) at A[i*lda + k], bf16
+ *   B: K x N, row-major, element (k, j) at B[k*ldb + j], bf16
+ *   C: M x N, row-major, element (i, j) at C[i*ldc + j], fp32 or bf16
+ *   C = A * B with fp32 accumulation; bf16 output is rounded to nearest even.
+ */
+#ifndef GOLDY_H_
+#define GOLDY_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GOLDY_ABI_VERSION 1
+
+typedef enum goldy_status {
+  GOLDY_OK = 0,
+  GOLDY_ERR_INVALID_ARG = 1,   /* null pointer, bad size, bad stride, bad flags */
+  GOLDY_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement */
+  GOLDY_ERR_LUT = 3,           /* lookup table missing, malformed or empty */
+  GOLDY_ERR_CUDA = 4,          /* a CUDA runtime/driver call failed */
+  GOLDY_ERR_TIMEOUT = 5,       /* a kernel gave up a bounded wait (see goldy_device_error) */
+  GOLDY_ERR_NOMEM = 6          /* host allocation failed, or a caller buffer is too small */
+} goldy_status;
+
+typedef enum goldy_dtype { GOLDY_BF16 = 0, GOLDY_F32 = 1 } goldy_dtype;
+
+/* One GEMM (Sec. 2.1.2).  Sizes and leading dimensions are in elements.
+ * Supported now: trans_a = trans_b = 0, a = b = GOLDY_BF16, c = BF16 or F32,
+ * M, N, K >= 0, lda >= K, ldb >= N, ldc >= N, lda and ldb multiples of 8
+ * (16-byte rows for the tensor-memory-accelerator copies). */
+typedef struct goldy_gemm_desc {
+  int64_t M, N, K;
+  int64_t lda, ldb, ldc;
+  int32_t trans_a, trans_b;    /* the paper's T1, T2; only 0, 0 is supported */
+  int32_t a_dtype, b_dtype, c_dtype;
+  int32_t reserved;            /* must be 0 */
+} goldy_gemm_desc;
+
+typedef struct goldy_lut goldy_lut;
+typedef struct goldy_schedule goldy_schedule;
+typedef struct goldy_graph goldy_graph;
+
+/* ---- planning policies (goldy_plan flags) -------------------------------
+ * The comparison configurations of Sec. 5.4 through one schedule type:
+ *   AUTO        the dynamic logic: preferred CD from the table, min(CD,
+ *               available), heterogeneous grouping (Sec. 4.3, Sec. 6.6)
+ *   SEQUENTIAL  isolation-tuned kernels one after another ("sequential")
+ *   DEFAULT     isolation-tuned kernels, every GEMM at once on its own stream
+ *               ("default", the naive all-streams launch)
+ *   GO          GO-Kernels for CD = n, every GEMM at once ("GO-Kernels")
+ *   FORCE_CD    GO-Kernels at a fixed CD; put the CD in bits 8..15
+ *               (GOLDY_PLAN_FORCE_CD | (cd << 8)) */
+#define GOLDY_PLAN_AUTO 0
+#define GOLDY_PLAN_SEQUENTIAL 1
+#define GOLDY_PLAN_DEFAULT 2
+#define GOLDY_PLAN_GO 3
+#define GOLDY_PLAN_FORCE_CD 4
+
+#define GOLDY_MAX_GEMMS 64      /* GEMMs per plan */
+#define GOLDY_MAX_STREAMS 16    /* concurrency degrees 1, 2, 4, 8, 16 (Sec. 4.3) */
+
+/* ---- version / device ---------------------------------------------------- */
+
+/* GOLDY_ABI_VERSION of the loaded library. */
+int goldy_abi_version(void);
+
+/* Text of the last error on this thread ("" if none).  Valid until the next
+ * call into the library from the same thread. */
+const char* goldy_last_error(void);
+
+/* ---- kernel variant registry --------------------------------------------
+ * A variant is one GO-Kernel configuration (Sec. 4.2): a tile shape and
+ * shared-memory/tensor-memory footprint (kind), a split of the K loop, and a
+ * resource constraint (RC) capping the persistent grid at the whole GPU, half
+ * or a quarter of it (Sec. 4.2.1's GPU, GPU/2, GPU/4). */
+typedef struct goldy_variant_info {
+  int32_t id;
+  int32_t kind;           /* tile/footprint family, 0 .. n_kinds-1 */
+  int32_t mma_m;          /* rows of the tensor-core tile (128) */
+  int32_t mma_n;          /* columns of the tensor-core tile */
+  int32_t swap_ab;        /* 1: computes C^T = B^T A^T tiles (skinny M) */
+  int32_t stages;         /* shared-memory pipeline depth */
+  int32_t acc_stages;     /* accumulators held in tensor memory */
+  int32_t tmem_cols;      /* tensor-memory columns allocated per CTA */
+  int32_t smem_bytes;     /* dynamic shared memory per CTA */
+  int32_t split_k;        /* K-loop split factor (1, 2, 4, 8) */
+  int32_t rc_div;         /* grid cap = resident CTAs per SM * SMs / rc_div */
+  int32_t ctas_per_sm;    /* CTAs per SM the footprint is sized for */
+  char name[32];
+} goldy_variant_info;
+
+/* Number of variant ids (ids are 0 .. count-1). */
+int goldy_variant_count(void);
+
+/* Describe variant `id`.  GOLDY_ERR_INVALID_ARG if id is out of range or out
+ * is null. */
+goldy_status goldy_variant_info_get(int id, goldy_variant_info* out);
+
+/* ---- lookup table (the dynamic logic's profiled data, Sec. 4.3) ---------
+ * File format (little-endian): magic "GOLDYLUT", u32 version = 1, u32 entry
+ * count, u32 variant-id bound, u32 SM count of the profiling GPU, 8 zero
+ * bytes; then 16-byte entries {u8 lm, ln, lk, out_dtype; u8 pref_cd; u8 0;
+ * u16 variant[5]} strictly sorted by (lm, ln, lk, out_dtype), where lm, ln,
+ * lk are floor(log2) of M, N, K and variant[c] is the GO-Kernel for CD class
+ * c in {1, 2, 4, 8, 16}.  GOLDY_ERR_LUT if the data is malformed or empty. */
+goldy_status goldy_lut_load(const char* path, goldy_lut** out);
+goldy_status goldy_lut_from_memory(const void* data, size_t bytes, goldy_lut** out);
+void goldy_lut_free(goldy_lut* lut);
+
+/* Bucket key of one GEMM: (lm << 24) | (ln << 16) | (lk << 8) | c_dtype,
+ * each log2 floored (0 for a size of 0) and clamped to 255. */
+goldy_status goldy_bucket_key(const goldy_gemm_desc* d, uint32_t* key);
+
+/* ---- planning (host only; makes no CUDA call) ---------------------------
+ * Plan n (1 .. GOLDY_MAX_GEMMS) GEMMs with the policy in `flags`.
+ * Deterministic: the schedule is a pure function of (descs, lut, flags).
+ * GOLDY_ERR_INVALID_ARG for null pointers, n out of range, bad flags or a
+ * descriptor violating the layout rules above; GOLDY_ERR_UNSUPPORTED for a
+ * transposed operand or unsupported dtype. */
+goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const goldy_lut* lut,
+                        int flags, goldy_schedule** out);
+
+/* Explicit schedule (used by the offline profiler and for measuring any
+ * chosen schedule): GEMM i runs in group group_of[i] (groups are run in
+ * increasing order, ids 0 .. n_groups-1 all used), with variant
+ * variant_of[i], on stream slot slot_of[i] (< GOLDY_MAX_STREAMS).  A group's
+ * CD is its number of distinct slots. */
+goldy_status goldy_schedule_build(const goldy_gemm_desc* descs, int n, const int* group_of,
+                                  const int* variant_of, const int* slot_of,
+                                  goldy_schedule** out);
+
+/* Sizes of a schedule.  workspace_bytes is the device workspace goldy_run
+ * needs (split-K partial tiles and arrival counters, 0 if none). */
+goldy_status goldy_schedule_query(const goldy_schedule* s, int* n_gemms, int* n_groups,
+                                  int* max_streams, size_t* workspace_bytes);
+
+/* Placement of GEMM `gemm`: its group, variant, stream slot and its group's CD. */
+goldy_status goldy_schedule_entry(const goldy_schedule* s, int gemm, int* group,
+                                  int* variant, int* slot, int* cd);
+
+/* Canonical bytes of the plan (little-endian u32 words): "GSCH", version 1,
+ * n_gemms, n_groups, max_streams, flags; per group: cd, size, members in
+ * launch order; per GEMM: group, variant, slot.  Writes at most `cap` bytes;
+ * *size gets the full length (GOLDY_ERR_NOMEM if cap is too small). */
+goldy_status goldy_schedule_serialize(const goldy_schedule* s, void* buf, size_t cap,
+                                      size_t* size);
+
+void goldy_schedule_free(goldy_schedule* s);
+
+/* ---- execution ----------------------------------------------------------
+ * Launch schedule `s`: A[i], B[i], C[i] are device pointers of GEMM i;
+ * `workspace` is a device buffer of at least goldy_schedule_query's
+ * workspace_bytes (may be null when that is 0), zero-filled by the caller
+ * before its first use — the kernels leave it zero-filled after every
+ * complete run; streams[0 .. n_streams-1] are CUDA streams with n_streams >=
+ * max_streams.  Groups run in order; a group forks from streams[0] and joins
+ * back to it, so work queued on streams[0] before the call happens before
+ * every GEMM and work queued on streams[0] after it happens after all of
+ * them.  Slot k runs on streams[k].  Asynchronous: returns after launching;
+ * no allocation, no synchronisation.  Errors: GOLDY_ERR_INVALID_ARG (null or
+ * misaligned pointers, too few streams, workspace too small),
+ * GOLDY_ERR_CUDA (launch failure).  A kernel that gave up a bounded wait
+ * shows up later through goldy_device_error(). */
+goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void* const* B,
+                       void* const* C, void* workspace, size_t workspace_bytes,
+                       void* const* streams, int n_streams);
+
+/* Capture goldy_run(...) with these exact pointers into a CUDA graph, for
+ * replay with one launch (the closest host-side analogue of the command
+ * processor dispatching a whole set).  The streams must be idle.  The graph
+ * owns copies of all launch parameters; the buffers must outlive it. */
+goldy_status goldy_graph_create(const goldy_schedule* s, const void* const* A,
+                                const void* const* B, void* const* C, void* workspace,
+                                size_t workspace_bytes, void* const* streams, int n_streams,
+                                goldy_graph** out);
+/* Launch a captured graph on `stream` (asynchronous). */
+goldy_status goldy_graph_launch(const goldy_graph* g, void* stream);
+void goldy_graph_free(goldy_graph* g);
+
+/* Error word the kernels set when a bounded wait gives up (0 = none).  Reads
+ * it synchronously on the current device and, if `clear`, resets it. */
+goldy_status goldy_device_error(int* code, int clear);
+
+/* SM count and CTAs of variant `variant_id` resident per SM on the current
+ * device (occupancy query, no launch). */
+goldy_status goldy_device_info(int variant_id, int* sm_count, int* ctas_per_sm);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GOLDY_H_ */

@@ -170,7 +170,7 @@ def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
         raise PlanError("bad count")
     policy = flags & 0xF
     forced = (flags >> 8) & 0xFF
-    if policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
+    if (flags & ~0xFF0F) or policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
         raise PlanError("bad flags")
     keys = [bucket_key(d.M, d.N, d.K, d.out_dtype) for d in descs]
     ents = [lookup(entries, k) for k in keys]

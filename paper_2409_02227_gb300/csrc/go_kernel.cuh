@@ -1,0 +1,436 @@
+// GO-Kernel: persistent, warp-specialised BF16 GEMM for sm_103a.
+//
+// What it computes (Sec. 2.1.2): C = A * B for A (M x K, row-major), B
+// (K x N, row-major), fp32 accumulation, fp32 or bf16 (round-to-nearest-even)
+// output.  Several GEMMs may share one launch (the launch's "units" are the
+// concatenation of their tiles).
+//
+// How (Sec. 2.1.3's tiled GEMM re-expressed for tcgen05):
+//   * The output is cut into tiles; a tile with its K-range split is a
+//     "unit".  CTA b processes units b, b + gridDim.x, ... (persistent CTAs,
+//     a static round-robin that is a function of the variant only).  The
+//     grid size is the variant's resource constraint: capping it is how a
+//     GO-Kernel leaves SMs to co-running GEMMs (Sec. 4.2.1).
+//   * warp 0 (one thread): TMA producer.  Per 64-wide K block it loads the
+//     A tile (K-major, 128-byte swizzle) and the B tile (N-major, 128-byte
+//     swizzle) into a shared-memory ring of STAGES slots (mbarrier full/empty).
+//   * warp 1 (one thread): allocates tensor memory, issues tcgen05.mma
+//     (M = 128, N = MMA_N, K = 16 per instruction) into an fp32 accumulator
+//     in tensor memory, ACC accumulators deep so the epilogue of one tile
+//     overlaps the main loop of the next.
+//   * warps 2-5: epilogue.  tcgen05.ld the accumulator (each warp its lane
+//     quarter), convert and store to C.  With split-K, each split writes its
+//     fp32 partial tile to the workspace; the last split to arrive (atomic
+//     counter, no waiting on other CTAs) adds the partials in split order
+//     0, 1, ..., S-1 and writes C, so every output element is summed in an
+//     order fixed by the variant alone: results are bit-identical whether
+//     the GEMM runs alone or next to others.
+//   * SWAP (skinny M): the tensor-core tile is C^T — the 128-row MMA operand
+//     is a slice of B's columns and the MMA_N-wide operand a slice of A's
+//     rows — so an M of 16..64 still fills the 128-row tensor-core shape.
+//
+// Every wait is bounded (sm103_ptx.cuh).  A role that gives up raises the
+// CTA's abort flag and the device error word, waits (bounded) for its own
+// copies or MMAs in flight, and the CTA frees its tensor memory and exits.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "sm103_ptx.cuh"
+
+namespace goldy {
+
+struct GemmWork {
+  void* c;              // output, row-major, ldc elements per row
+  float* ws_part;       // split-K partial tiles (null when split == 1)
+  uint32_t* ws_cnt;     // split-K arrival counter per tile
+  int64_t ldc;
+  int32_t m, n, k;
+  int32_t tiles_m, tiles_n;
+  int32_t split;        // K-range split, 1 <= split <= k_blocks
+  int32_t k_blocks;     // ceil(K / 64)
+  int32_t unit_begin;   // first unit of this GEMM within the launch
+  int32_t pad_[3];
+};
+
+template <int MAXG>
+struct LaunchParams {
+  CUtensorMap tmap_a[MAXG];   // A: dims {K, M}, box {64, rows of the A tile}
+  CUtensorMap tmap_b[MAXG];   // B: dims {N, K}, box {64, 64}
+  GemmWork g[MAXG];
+  int32_t n_gemms;
+  int32_t total_units;
+  int* err;                   // device error word (first failure wins)
+};
+
+enum : int {
+  kErrProducerWait = 1,
+  kErrMmaWait = 2,
+  kErrEpilogueWait = 3,
+};
+
+struct UnitCoord {
+  int g, tile, s, tm, tn, kb0, kb1;
+};
+
+template <int MAXG>
+__device__ __forceinline__ UnitCoord decode_unit(const LaunchParams<MAXG>& p, int u) {
+  UnitCoord c;
+  int g = 0;
+#pragma unroll 1
+  while (g + 1 < p.n_gemms && u >= p.g[g + 1].unit_begin) ++g;
+  const GemmWork& w = p.g[g];
+  const int local = u - w.unit_begin;
+  c.g = g;
+  c.tile = local / w.split;
+  c.s = local - c.tile * w.split;
+  c.tm = c.tile % w.tiles_m;
+  c.tn = c.tile / w.tiles_m;
+  c.kb0 = (c.s * w.k_blocks) / w.split;
+  c.kb1 = ((c.s + 1) * w.k_blocks) / w.split;
+  return c;
+}
+
+__device__ __forceinline__ void raise_error(int* err, volatile int* abort_flag, int code) {
+  *abort_flag = 1;
+  if (err) atomicCAS(err, 0, code);
+}
+
+// Store 32 consecutive accumulator columns of one accumulator row.
+//  !SWAP: row `r` of the tile is C row m0 + r; columns n0 + c0 .. +31.
+//   SWAP: row `r` of the tile is C column n0 + r; columns are C rows m0 + c0 .. +31.
+template <bool SWAP, bool OUT_BF16>
+__device__ __forceinline__ void store_chunk(const GemmWork& w, int m0, int n0, int r, int c0, const float (&v)[32]) {
+  if (!SWAP) {
+    const int64_t row = int64_t(m0) + r;
+    if (row >= w.m) return;
+    const int col0 = n0 + c0;
+    if (OUT_BF16) {
+      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(w.c) + row * w.ldc + col0;
+      if (col0 + 32 <= w.n && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint4 pk;
+          __nv_bfloat162 h0 = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
+          __nv_bfloat162 h1 = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
+          __nv_bfloat162 h3 = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
+          pk.x = *reinterpret_cast<uint32_t*>(&h0);
+          pk.y = *reinterpret_cast<uint32_t*>(&h1);
+          pk.z = *reinterpret_cast<uint32_t*>(&h2);
+          pk.w = *reinterpret_cast<uint32_t*>(&h3);
+          reinterpret_cast<uint4*>(dst)[q] = pk;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (col0 + j < w.n) dst[j] = __float2bfloat16_rn(v[j]);
+      }
+    } else {
+      float* dst = static_cast<float*>(w.c) + row * w.ldc + col0;
+      if (col0 + 32 <= w.n && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          reinterpret_cast<float4*>(dst)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (col0 + j < w.n) dst[j] = v[j];
+      }
+    }
+  } else {
+    const int64_t col = int64_t(n0) + r;
+    if (col >= w.n) return;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int64_t row = int64_t(m0) + c0 + j;
+      if (row < w.m) {
+        if (OUT_BF16)
+          static_cast<__nv_bfloat16*>(w.c)[row * w.ldc + col] = __float2bfloat16_rn(v[j]);
+        else
+          static_cast<float*>(w.c)[row * w.ldc + col] = v[j];
+      }
+    }
+  }
+}
+
+template <int MMA_N, int ACC>
+struct TmemCols {
+  static constexpr uint32_t need = uint32_t(MMA_N * ACC);
+  static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
+};
+
+template <int MMA_N, bool SWAP, int STAGES, int ACC, bool OUT_BF16, int MAXG>
+__global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__ LaunchParams<MAXG> p) {
+  constexpr int X_BYTES = 128 * 64 * 2;              // MMA operand A: 128 rows x 64 K
+  constexpr int Y_BYTES = MMA_N * 64 * 2;            // MMA operand B: MMA_N rows x 64 K
+  constexpr int STAGE_BYTES = X_BYTES + Y_BYTES;
+  constexpr int TILE_M = SWAP ? MMA_N : 128;         // C rows per tile
+  constexpr int TILE_N = SWAP ? 128 : MMA_N;         // C columns per tile
+  constexpr int B_BOXES = TILE_N / 64;               // 64-column TMA boxes of B per stage
+  constexpr uint32_t TMEM_COLS = TmemCols<MMA_N, ACC>::value;
+  // !SWAP: MMA-A = A tile (K-major), MMA-B = B tile (N-major)
+  //  SWAP: MMA-A = B tile (N-major), MMA-B = A tile (K-major)
+  constexpr uint32_t IDESC = ptx::make_idesc_bf16(128, MMA_N, SWAP ? 1 : 0, SWAP ? 0 : 1);
+  constexpr uint32_t KMAJ_STEP = 32;                 // bytes per 16 K elements, K-major
+  constexpr uint32_t MNMAJ_STEP = 2048;              // bytes per 16 K rows, N-major
+  constexpr uint32_t MNMAJ_LBO = 64 * 128;           // bytes between 64-wide N chunks
+  static_assert(MMA_N % 32 == 0 && MMA_N >= 32 && MMA_N <= 256, "MMA_N");
+  static_assert(TILE_N % 64 == 0, "B tiles are whole 64-column boxes");
+  static_assert(STAGES <= 32, "stage bitmasks");
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* tfull = bars + 2 * STAGES;
+  uint64_t* tempty = bars + 2 * STAGES + ACC;
+  uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
+
+  const uint32_t tiles_base = ptx::smem_u32(smem);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      ptx::mbar_init(ptx::smem_u32(&full[s]), 1);
+      ptx::mbar_init(ptx::smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < ACC; ++a) {
+      ptx::mbar_init(ptx::smem_u32(&tfull[a]), 1);
+      ptx::mbar_init(ptx::smem_u32(&tempty[a]), 128);
+    }
+    ptx::mbar_init(ptx::smem_u32(drain), 1);
+    *abort_flag = 0;
+    *last_flag = 0;
+    ptx::fence_barrier_init();
+    ptx::fence_proxy_async_smem();
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(ptx::smem_u32(tmem_slot), TMEM_COLS);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ producer
+      for (int g = 0; g < p.n_gemms; ++g) {
+        ptx::prefetch_tensormap(&p.tmap_a[g]);
+        ptx::prefetch_tensormap(&p.tmap_b[g]);
+      }
+      int stage = 0;
+      uint32_t phase = 0, issued = 0, last_phase = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
+        const UnitCoord c = decode_unit(p, u);
+        const void* ta = &p.tmap_a[c.g];
+        const void* tb = &p.tmap_b[c.g];
+        const int m0 = c.tm * TILE_M;
+        const int n0 = c.tn * TILE_N;
+        for (int kb = c.kb0; kb < c.kb1; ++kb) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = ptx::smem_u32(&full[stage]);
+          ptx::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+          const uint32_t xs = tiles_base + stage * STAGE_BYTES;
+          const uint32_t ys = xs + X_BYTES;
+          const int k0 = kb * 64;
+          if (!SWAP) {
+            ptx::tma_load_2d(xs, ta, fb, k0, m0);
+#pragma unroll
+            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_2d(ys + j * 8192, tb, fb, n0 + 64 * j, k0);
+          } else {
+#pragma unroll
+            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_2d(xs + j * 8192, tb, fb, n0 + 64 * j, k0);
+            ptx::tma_load_2d(ys, ta, fb, k0, m0);
+          }
+          issued |= 1u << stage;
+          last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (!ok) {
+        raise_error(p.err, abort_flag, kErrProducerWait);
+        // let every copy this thread started land before the CTA can exit
+        for (int s = 0; s < STAGES; ++s)
+          if (issued >> s & 1) ptx::mbar_wait(ptx::smem_u32(&full[s]), (last_phase >> s) & 1, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------- MMA issuer
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true, any = false;
+      for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
+        const UnitCoord c = decode_unit(p, u);
+        if (!ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + uint32_t(acc * MMA_N);
+        for (int kb = c.kb0; kb < c.kb1; ++kb) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          const uint32_t xs = tiles_base + stage * STAGE_BYTES;
+          const uint32_t ys = xs + X_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            uint64_t adesc, bdesc;
+            if (!SWAP) {
+              adesc = ptx::make_sdesc_sw128(xs + kk * KMAJ_STEP, 16, 1024);
+              bdesc = ptx::make_sdesc_sw128(ys + kk * MNMAJ_STEP, MNMAJ_LBO, 1024);
+            } else {
+              adesc = ptx::make_sdesc_sw128(xs + kk * MNMAJ_STEP, MNMAJ_LBO, 1024);
+              bdesc = ptx::make_sdesc_sw128(ys + kk * KMAJ_STEP, 16, 1024);
+            }
+            ptx::mma_bf16(d_tmem, adesc, bdesc, IDESC, (kb > c.kb0 || kk > 0) ? 1u : 0u);
+          }
+          any = true;
+          ptx::mma_commit(ptx::smem_u32(&empty[stage]));   // frees the slot when these MMAs finish
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        ptx::mma_commit(ptx::smem_u32(&tfull[acc]));        // accumulator complete
+        if (++acc == ACC) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
+      }
+      if (!ok) {
+        raise_error(p.err, abort_flag, kErrMmaWait);
+        if (any) {
+          ptx::mma_commit(ptx::smem_u32(drain));
+          ptx::mbar_wait(ptx::smem_u32(drain), 0, nullptr);
+        }
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue
+    const int q = warp & 3;                 // tensor-memory lane quarter of this warp
+    const int r = q * 32 + lane;            // accumulator row handled by this thread
+    const int et = threadIdx.x - 64;        // 0 .. 127
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
+      const UnitCoord c = decode_unit(p, u);
+      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
+      ok = ptx::named_bar_and(1, 128, ok);
+      if (!ok) {
+        if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
+        break;
+      }
+      ptx::tc_fence_after();
+      const GemmWork& w = p.g[c.g];
+      const int m0 = c.tm * TILE_M;
+      const int n0 = c.tn * TILE_N;
+      const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);
+      if (w.split == 1) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
+          store_chunk<SWAP, OUT_BF16>(w, m0, n0, r, c0, v);
+        }
+      } else {
+        // partial tile layout: [chunk][float4 index j4][row r] -> coalesced per warp
+        constexpr int TILE_F4 = 128 * MMA_N / 4;
+        float4* part_base = reinterpret_cast<float4*>(w.ws_part);
+        float4* mine = part_base + size_t(c.tile * w.split + c.s) * TILE_F4;
+#pragma unroll 1
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int j4 = 0; j4 < 8; ++j4)
+            mine[((c0 / 4) + j4) * 128 + r] =
+                make_float4(__uint_as_float(raw[4 * j4]), __uint_as_float(raw[4 * j4 + 1]),
+                            __uint_as_float(raw[4 * j4 + 2]), __uint_as_float(raw[4 * j4 + 3]));
+        }
+        __threadfence();
+        ptx::named_bar_sync(1, 128);
+        if (et == 0) {
+          const uint32_t old = atomicAdd(&w.ws_cnt[c.tile], 1u);
+          *last_flag = (old == uint32_t(w.split - 1)) ? 1 : 0;
+        }
+        ptx::named_bar_sync(1, 128);
+        if (*last_flag) {
+          __threadfence();
+#pragma unroll 1
+          for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+            uint32_t raw[32];
+            __syncwarp();
+            ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+            ptx::tmem_ld_wait();
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+#pragma unroll 1
+            for (int s2 = 0; s2 < w.split; ++s2) {
+              if (s2 == c.s) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(raw[j]);
+              } else {
+                const float4* other = part_base + size_t(c.tile * w.split + s2) * TILE_F4;
+#pragma unroll
+                for (int j4 = 0; j4 < 8; ++j4) {
+                  const float4 t = __ldcg(&other[((c0 / 4) + j4) * 128 + r]);
+                  v[4 * j4] += t.x;
+                  v[4 * j4 + 1] += t.y;
+                  v[4 * j4 + 2] += t.z;
+                  v[4 * j4 + 3] += t.w;
+                }
+              }
+            }
+            store_chunk<SWAP, OUT_BF16>(w, m0, n0, r, c0, v);
+          }
+          if (et == 0) w.ws_cnt[c.tile] = 0u;     // leave the counter zeroed for the next run
+        }
+      }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));
+      if (++acc == ACC) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace goldy

@@ -1,0 +1,353 @@
+// Launch manager: runs a schedule on caller-owned streams.
+//
+// The paper's command processor dispatches the chosen GEMMs from their queue
+// heads, as many at once as the predicted concurrency degree allows
+// (Sec. 4.4).  Here each group of the schedule forks from streams[0] with an
+// event, launches its GEMMs round-robin onto the group's stream slots (so at
+// most CD GEMMs are in flight, each stream running its GEMMs back to back),
+// and joins back into streams[0] before the next group starts.  The whole
+// run can be captured once into a CUDA graph and replayed with one launch.
+//
+// Per GEMM the host encodes two TMA tensor maps (A and B), sizes the
+// persistent grid as min(units, resident CTAs per SM * SMs / rc_div) — the
+// variant's resource constraint — and launches the kind's kernel.  Nothing
+// here allocates device memory or synchronises.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "go_kernel.cuh"
+#include "goldy_internal.h"
+
+namespace goldy {
+
+__device__ int g_device_error;   // kernels' error word (first failure wins)
+
+struct Runtime {
+  int device = -1;
+  cudaEvent_t fork = nullptr;
+  cudaEvent_t join[GOLDY_MAX_STREAMS] = {};
+};
+
+void runtime_release(Runtime* rt) {
+  if (!rt) return;
+  if (rt->fork) cudaEventDestroy(rt->fork);
+  for (cudaEvent_t e : rt->join)
+    if (e) cudaEventDestroy(e);
+  delete rt;
+}
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+  bool init = false;
+  int sm_count = 0;
+  int* err_word = nullptr;
+  int ctas_per_sm[kNumKinds][2] = {};   // 0 = not yet set up
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+goldy_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(GOLDY_ERR_CUDA, std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")");
+}
+
+const void* kernel_fn(int kind, int out_bf16) {
+  switch (kind) {
+    case 0: return kernel_fn_k0(out_bf16);
+    case 1: return kernel_fn_k1(out_bf16);
+    case 2: return kernel_fn_k2(out_bf16);
+    case 3: return kernel_fn_k3(out_bf16);
+    case 4: return kernel_fn_k4(out_bf16);
+    case 5: return kernel_fn_k5(out_bf16);
+    case 6: return kernel_fn_k6(out_bf16);
+    case 7: return kernel_fn_k7(out_bf16);
+    case 8: return kernel_fn_k8(out_bf16);
+    case 9: return kernel_fn_k9(out_bf16);
+    default: return nullptr;
+  }
+}
+
+// Per-device setup: SM count, error word address, encode entry point.
+goldy_status device_state(DeviceState** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(GOLDY_ERR_UNSUPPORTED, "device index too large");
+  std::lock_guard<std::mutex> lock(g_mu);
+  DeviceState& d = g_dev[dev];
+  if (!d.init) {
+    e = cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err_word), g_device_error);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+    if (!g_encode) {
+      cudaDriverEntryPointQueryResult q;
+      void* fn = nullptr;
+      e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+      if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return fail(GOLDY_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    d.init = true;
+  }
+  *out = &d;
+  return GOLDY_OK;
+}
+
+// Resident CTAs per SM of one kernel (kind, dtype) on this device; also opts
+// the kernel into its dynamic shared-memory size the first time.
+goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int* ctas) {
+  std::lock_guard<std::mutex> lock(g_mu);
+  int& c = d.ctas_per_sm[kind][out_bf16];
+  if (c == 0) {
+    const void* fn = kernel_fn(kind, out_bf16);
+    if (!fn) return fail(GOLDY_ERR_UNSUPPORTED, "no kernel for this kind");
+    const KindInfo& k = kKinds[kind];
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes(k));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+    int occ = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, kThreads, smem_bytes(k));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+    // tensor memory is not part of the occupancy query: 512 columns per SM
+    occ = std::min(occ, 512 / tmem_cols(k));
+    if (occ < 1) return fail(GOLDY_ERR_UNSUPPORTED, "kernel does not fit on an SM");
+    c = occ;
+  }
+  *ctas = c;
+  return GOLDY_OK;
+}
+
+goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                       uint32_t box_inner, uint32_t box_outer) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuTensorMapEncodeTiled failed with code " + std::to_string(int(r)));
+  return GOLDY_OK;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, const void* B, void* C, uint8_t* ws,
+                         cudaStream_t stream) {
+  const goldy_gemm_desc& g = gp.desc;
+  const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
+  if (g.M == 0 || g.N == 0) return GOLDY_OK;
+  if (g.K == 0) {
+    cudaError_t e = cudaMemset2DAsync(C, size_t(g.ldc) * es, 0, size_t(g.N) * es, size_t(g.M), stream);
+    return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
+  }
+  const KindInfo& k = kKinds[gp.kind];
+  const int out_bf16 = g.c_dtype == GOLDY_BF16 ? 1 : 0;
+  int ctas = 0;
+  goldy_status st = kernel_setup(d, gp.kind, out_bf16, &ctas);
+  if (st != GOLDY_OK) return st;
+
+  LaunchParams<1> p;
+  std::memset(&p, 0, sizeof(p));
+  st = encode_2d(&p.tmap_a[0], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(tile_rows(k)));
+  if (st != GOLDY_OK) return st;
+  st = encode_2d(&p.tmap_b[0], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.ldb) * 2, 64, kBlockK);
+  if (st != GOLDY_OK) return st;
+  GemmWork& w = p.g[0];
+  w.c = C;
+  w.ldc = g.ldc;
+  w.m = int32_t(g.M);
+  w.n = int32_t(g.N);
+  w.k = int32_t(g.K);
+  w.tiles_m = int32_t(gp.tiles_m);
+  w.tiles_n = int32_t(gp.tiles_n);
+  w.split = gp.split;
+  w.k_blocks = int32_t(gp.k_blocks);
+  w.unit_begin = 0;
+  if (gp.split > 1) {
+    w.ws_part = reinterpret_cast<float*>(ws + gp.ws_part_off);
+    w.ws_cnt = reinterpret_cast<uint32_t*>(ws + gp.ws_cnt_off);
+  }
+  p.n_gemms = 1;
+  if (gp.units > int64_t(1) << 30) return fail(GOLDY_ERR_UNSUPPORTED, "too many tiles in one GEMM");
+  p.total_units = int32_t(gp.units);
+  p.err = d.err_word;
+
+  const Variant v = variant_of(gp.variant);
+  const int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
+  const unsigned grid = unsigned(std::min<int64_t>(gp.units, cap));
+  void* args[] = {&p};
+  cudaError_t e = cudaLaunchKernel(kernel_fn(gp.kind, out_bf16), dim3(grid), dim3(kThreads), args,
+                                   size_t(smem_bytes(k)), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel");
+  return GOLDY_OK;
+}
+
+}  // namespace
+}  // namespace goldy
+
+using namespace goldy;
+
+extern "C" goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                  void* const* C, void* workspace, size_t workspace_bytes, void* const* streams,
+                                  int n_streams) {
+  if (!s || !A || !B || !C || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  if (n_streams < s->max_streams) return fail(GOLDY_ERR_INVALID_ARG, "fewer streams than the schedule needs");
+  if (s->workspace_bytes > 0) {
+    if (!workspace || workspace_bytes < s->workspace_bytes)
+      return fail(GOLDY_ERR_INVALID_ARG, "workspace missing or smaller than goldy_schedule_query reports");
+    if (!aligned(workspace, 256)) return fail(GOLDY_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  }
+  for (size_t i = 0; i < s->gemms.size(); ++i) {
+    const goldy_gemm_desc& g = s->gemms[i].desc;
+    if (g.M == 0 || g.N == 0) continue;
+    const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
+    if (!C[i] || !aligned(C[i], es)) return fail(GOLDY_ERR_INVALID_ARG, "gemm " + std::to_string(i) + ": C null or misaligned");
+    if (g.K == 0) continue;
+    if (!A[i] || !B[i] || !aligned(A[i], 16) || !aligned(B[i], 16))
+      return fail(GOLDY_ERR_INVALID_ARG, "gemm " + std::to_string(i) + ": A and B must be 16-byte aligned device pointers");
+  }
+  DeviceState* d = nullptr;
+  goldy_status st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+
+  goldy_schedule* ms = const_cast<goldy_schedule*>(s);
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (ms->rt && ms->rt->device != dev) {
+    runtime_release(ms->rt);
+    ms->rt = nullptr;
+  }
+  if (!ms->rt) {
+    Runtime* rt = new Runtime();
+    rt->device = dev;
+    cudaError_t e = cudaEventCreateWithFlags(&rt->fork, cudaEventDisableTiming);
+    for (int k = 0; k < GOLDY_MAX_STREAMS && e == cudaSuccess; ++k)
+      e = cudaEventCreateWithFlags(&rt->join[k], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      runtime_release(rt);
+      return cuda_fail(e, "cudaEventCreate");
+    }
+    ms->rt = rt;
+  }
+  Runtime* rt = ms->rt;
+  cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+
+  for (const Group& grp : s->groups) {
+    uint32_t used = 0;
+    for (int i : grp.members) used |= 1u << s->gemms[i].slot;
+    const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
+    if (side) {
+      cudaError_t e = cudaEventRecord(rt->fork, main);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+      for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
+        if (side >> k & 1) {
+          e = cudaStreamWaitEvent(static_cast<cudaStream_t>(streams[k]), rt->fork, 0);
+          if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+        }
+    }
+    for (int i : grp.members) {
+      const GemmPlan& gp = s->gemms[i];
+      st = launch_gemm(*d, gp, A[i], B[i], C[i], ws, static_cast<cudaStream_t>(streams[gp.slot]));
+      if (st != GOLDY_OK) return st;
+    }
+    if (side) {
+      for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
+        if (side >> k & 1) {
+          cudaError_t e = cudaEventRecord(rt->join[k], static_cast<cudaStream_t>(streams[k]));
+          if (e == cudaSuccess) e = cudaStreamWaitEvent(main, rt->join[k], 0);
+          if (e != cudaSuccess) return cuda_fail(e, "join event");
+        }
+    }
+  }
+  return ok();
+}
+
+struct goldy_graph {
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+};
+
+extern "C" goldy_status goldy_graph_create(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                           void* const* C, void* workspace, size_t workspace_bytes,
+                                           void* const* streams, int n_streams, goldy_graph** out) {
+  if (!out || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
+  cudaError_t e = cudaStreamBeginCapture(main, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamBeginCapture");
+  goldy_status st = goldy_run(s, A, B, C, workspace, workspace_bytes, streams, n_streams);
+  std::string why = st == GOLDY_OK ? "" : goldy_last_error();
+  cudaGraph_t graph = nullptr;
+  e = cudaStreamEndCapture(main, &graph);
+  if (st != GOLDY_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return fail(st, why);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamEndCapture");
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  if (e != cudaSuccess) {
+    cudaGraphDestroy(graph);
+    return cuda_fail(e, "cudaGraphInstantiate");
+  }
+  goldy_graph* g = new goldy_graph();
+  g->graph = graph;
+  g->exec = exec;
+  *out = g;
+  return ok();
+}
+
+extern "C" goldy_status goldy_graph_launch(const goldy_graph* g, void* stream) {
+  if (!g) return fail(GOLDY_ERR_INVALID_ARG, "null graph");
+  cudaError_t e = cudaGraphLaunch(g->exec, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
+  return ok();
+}
+
+extern "C" void goldy_graph_free(goldy_graph* g) {
+  if (!g) return;
+  if (g->exec) cudaGraphExecDestroy(g->exec);
+  if (g->graph) cudaGraphDestroy(g->graph);
+  delete g;
+}
+
+extern "C" goldy_status goldy_device_error(int* code, int clear) {
+  if (!code) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  DeviceState* d = nullptr;
+  goldy_status st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+  cudaError_t e = cudaMemcpy(code, d->err_word, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy (error word)");
+  if (clear && *code != 0) {
+    const int zero = 0;
+    e = cudaMemcpy(d->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy (clear error word)");
+  }
+  return ok();
+}
+
+extern "C" goldy_status goldy_device_info(int variant_id, int* sm_count, int* ctas_per_sm) {
+  if (variant_id < 0 || variant_id >= kNumVariants) return fail(GOLDY_ERR_INVALID_ARG, "variant id out of range");
+  DeviceState* d = nullptr;
+  goldy_status st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+  const Variant v = variant_of(variant_id);
+  int ctas = 0;
+  st = kernel_setup(*d, v.kind, 0, &ctas);
+  if (st != GOLDY_OK) return st;
+  if (sm_count) *sm_count = d->sm_count;
+  if (ctas_per_sm) *ctas_per_sm = ctas;
+  return ok();
+}

@@ -1,0 +1,293 @@
+"""ctypes binding of ``include/goldy.h`` — argument marshalling only.
+
+Every function here has the name of the C entry point it calls and does no
+work of its own beyond converting arguments and raising ``GoldyError`` on a
+non-zero status.  Device pointers and CUDA streams are plain integers
+(``tensor.data_ptr()``, ``torch.cuda.Stream().cuda_stream``).  The library is
+``libgoldy.so`` next to this file, built by ``paper_2409_02227_gb300.build``;
+importing this module without it raises ImportError — there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence, Tuple
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libgoldy.so")
+DEFAULT_LUT = os.path.join(_HERE, "data", "goldy_lut.bin")
+
+GOLDY_OK = 0
+GOLDY_ERR_INVALID_ARG = 1
+GOLDY_ERR_UNSUPPORTED = 2
+GOLDY_ERR_LUT = 3
+GOLDY_ERR_CUDA = 4
+GOLDY_ERR_TIMEOUT = 5
+GOLDY_ERR_NOMEM = 6
+
+GOLDY_BF16 = 0
+GOLDY_F32 = 1
+
+GOLDY_PLAN_AUTO = 0
+GOLDY_PLAN_SEQUENTIAL = 1
+GOLDY_PLAN_DEFAULT = 2
+GOLDY_PLAN_GO = 3
+GOLDY_PLAN_FORCE_CD = 4
+GOLDY_MAX_GEMMS = 64
+GOLDY_MAX_STREAMS = 16
+
+
+def force_cd(cd: int) -> int:
+    """Flags for GOLDY_PLAN_FORCE_CD with concurrency degree ``cd``."""
+    return GOLDY_PLAN_FORCE_CD | (int(cd) << 8)
+
+
+class GoldyError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str):
+        super().__init__(f"{where}: status {status}: {message}")
+        self.status = status
+
+
+class goldy_gemm_desc(ctypes.Structure):
+    _fields_ = [("M", ctypes.c_int64), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
+                ("lda", ctypes.c_int64), ("ldb", ctypes.c_int64), ("ldc", ctypes.c_int64),
+                ("trans_a", ctypes.c_int32), ("trans_b", ctypes.c_int32),
+                ("a_dtype", ctypes.c_int32), ("b_dtype", ctypes.c_int32),
+                ("c_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class goldy_variant_info(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("id", "kind", "mma_m", "mma_n", "swap_ab", "stages", "acc_stages", "tmem_cols",
+                 "smem_bytes", "split_k", "rc_div", "ctas_per_sm")] + [("name", ctypes.c_char * 32)]
+
+    def as_dict(self) -> dict:
+        d = {n: getattr(self, n) for n, _ in self._fields_ if n != "name"}
+        d["name"] = self.name.decode()
+        return d
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with "
+                          "`python -c 'import __graft_entry__ as g; g.build()'` (no CPU fallback exists)")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, U32, SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint32, ctypes.c_size_t
+    PP = ctypes.POINTER(ctypes.c_void_p)
+    IP = ctypes.POINTER(ctypes.c_int)
+    DP = ctypes.POINTER(goldy_gemm_desc)
+    sig = {
+        "goldy_abi_version": ([], I),
+        "goldy_last_error": ([], ctypes.c_char_p),
+        "goldy_variant_count": ([], I),
+        "goldy_variant_info_get": ([I, ctypes.POINTER(goldy_variant_info)], I),
+        "goldy_lut_load": ([ctypes.c_char_p, PP], I),
+        "goldy_lut_from_memory": ([P, SZ, PP], I),
+        "goldy_lut_free": ([P], None),
+        "goldy_bucket_key": ([DP, ctypes.POINTER(U32)], I),
+        "goldy_plan": ([DP, I, P, I, PP], I),
+        "goldy_schedule_build": ([DP, I, IP, IP, IP, PP], I),
+        "goldy_schedule_query": ([P, IP, IP, IP, ctypes.POINTER(SZ)], I),
+        "goldy_schedule_entry": ([P, I, IP, IP, IP, IP], I),
+        "goldy_schedule_serialize": ([P, P, SZ, ctypes.POINTER(SZ)], I),
+        "goldy_schedule_free": ([P], None),
+        "goldy_run": ([P, PP, PP, PP, P, SZ, PP, I], I),
+        "goldy_graph_create": ([P, PP, PP, PP, P, SZ, PP, I, PP], I),
+        "goldy_graph_launch": ([P, P], I),
+        "goldy_graph_free": ([P], None),
+        "goldy_device_error": ([IP, I], I),
+        "goldy_device_info": ([I, IP, IP], I),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    return lib
+
+
+_lib = _load()
+
+
+def _check(status: int, where: str) -> None:
+    if status != GOLDY_OK:
+        raise GoldyError(status, where, _lib.goldy_last_error().decode())
+
+
+def _ptrs(values: Sequence[int]):
+    arr = (ctypes.c_void_p * max(1, len(values)))()
+    for i, v in enumerate(values):
+        arr[i] = int(v) if v else None
+    return arr
+
+
+def _descs(descs: Sequence[goldy_gemm_desc]):
+    arr = (goldy_gemm_desc * max(1, len(descs)))()
+    for i, d in enumerate(descs):
+        arr[i] = d
+    return arr
+
+
+def desc(M: int, N: int, K: int, c_dtype: int = GOLDY_F32, lda: Optional[int] = None,
+         ldb: Optional[int] = None, ldc: Optional[int] = None) -> goldy_gemm_desc:
+    """Descriptor of C (M x N) = A (M x K, row-major) * B (K x N, row-major)."""
+    return goldy_gemm_desc(M, N, K, K if lda is None else lda, N if ldb is None else ldb,
+                           N if ldc is None else ldc, 0, 0, GOLDY_BF16, GOLDY_BF16, int(c_dtype), 0)
+
+
+class _Handle:
+    _free = None
+
+    def __init__(self, ptr: ctypes.c_void_p):
+        self.ptr = ptr
+
+    def close(self) -> None:
+        if self.ptr:
+            type(self)._free(self.ptr)
+            self.ptr = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Lut(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_lut_free(p))
+
+
+class Schedule(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_schedule_free(p))
+
+
+class Graph(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_graph_free(p))
+
+
+def goldy_abi_version() -> int:
+    return int(_lib.goldy_abi_version())
+
+
+def goldy_last_error() -> str:
+    return _lib.goldy_last_error().decode()
+
+
+def goldy_variant_count() -> int:
+    return int(_lib.goldy_variant_count())
+
+
+def goldy_variant_info_get(variant_id: int) -> dict:
+    info = goldy_variant_info()
+    _check(_lib.goldy_variant_info_get(int(variant_id), ctypes.byref(info)), "goldy_variant_info_get")
+    return info.as_dict()
+
+
+def goldy_lut_load(path: str = DEFAULT_LUT) -> Lut:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_lut_load(path.encode(), ctypes.byref(out)), "goldy_lut_load")
+    return Lut(out)
+
+
+def goldy_lut_from_memory(data: bytes) -> Lut:
+    out = ctypes.c_void_p()
+    buf = ctypes.create_string_buffer(bytes(data), len(data))
+    _check(_lib.goldy_lut_from_memory(buf, len(data), ctypes.byref(out)), "goldy_lut_from_memory")
+    return Lut(out)
+
+
+def goldy_bucket_key(d: goldy_gemm_desc) -> int:
+    key = ctypes.c_uint32()
+    _check(_lib.goldy_bucket_key(ctypes.byref(d), ctypes.byref(key)), "goldy_bucket_key")
+    return int(key.value)
+
+
+def goldy_plan(descs: Sequence[goldy_gemm_desc], lut: Lut, flags: int = GOLDY_PLAN_AUTO) -> Schedule:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_plan(_descs(descs), len(descs), lut.ptr if lut else None, int(flags),
+                           ctypes.byref(out)), "goldy_plan")
+    return Schedule(out)
+
+
+def goldy_schedule_build(descs: Sequence[goldy_gemm_desc], group_of: Sequence[int],
+                         variant_of: Sequence[int], slot_of: Sequence[int]) -> Schedule:
+    n = len(descs)
+    IA = ctypes.c_int * max(1, n)
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_schedule_build(_descs(descs), n, IA(*group_of), IA(*variant_of), IA(*slot_of),
+                                     ctypes.byref(out)), "goldy_schedule_build")
+    return Schedule(out)
+
+
+def goldy_schedule_query(s: Schedule) -> Tuple[int, int, int, int]:
+    """(n_gemms, n_groups, max_streams, workspace_bytes)."""
+    a, b, c, w = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_size_t()
+    _check(_lib.goldy_schedule_query(s.ptr, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c),
+                                     ctypes.byref(w)), "goldy_schedule_query")
+    return a.value, b.value, c.value, int(w.value)
+
+
+def goldy_schedule_entry(s: Schedule, gemm: int) -> Tuple[int, int, int, int]:
+    """(group, variant, slot, cd) of GEMM ``gemm``."""
+    g, v, sl, cd = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(_lib.goldy_schedule_entry(s.ptr, int(gemm), ctypes.byref(g), ctypes.byref(v),
+                                     ctypes.byref(sl), ctypes.byref(cd)), "goldy_schedule_entry")
+    return g.value, v.value, sl.value, cd.value
+
+
+def goldy_schedule_serialize(s: Schedule) -> bytes:
+    size = ctypes.c_size_t()
+    _lib.goldy_schedule_serialize(s.ptr, None, 0, ctypes.byref(size))
+    buf = ctypes.create_string_buffer(size.value)
+    _check(_lib.goldy_schedule_serialize(s.ptr, buf, size.value, ctypes.byref(size)),
+           "goldy_schedule_serialize")
+    return buf.raw[:size.value]
+
+
+def goldy_run(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
+              workspace_bytes: int, streams: Sequence[int]) -> None:
+    _check(_lib.goldy_run(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
+                          int(workspace_bytes), _ptrs(streams), len(streams)), "goldy_run")
+
+
+def goldy_graph_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int],
+                       workspace: int, workspace_bytes: int, streams: Sequence[int]) -> Graph:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_graph_create(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
+                                   int(workspace_bytes), _ptrs(streams), len(streams),
+                                   ctypes.byref(out)), "goldy_graph_create")
+    return Graph(out)
+
+
+def goldy_graph_launch(g: Graph, stream: int) -> None:
+    _check(_lib.goldy_graph_launch(g.ptr, int(stream) or None), "goldy_graph_launch")
+
+
+def goldy_device_error(clear: bool = True) -> int:
+    code = ctypes.c_int()
+    _check(_lib.goldy_device_error(ctypes.byref(code), 1 if clear else 0), "goldy_device_error")
+    return code.value
+
+
+def goldy_device_info(variant_id: int = 0) -> Tuple[int, int]:
+    """(SM count, resident CTAs per SM of the variant's kernel)."""
+    sm, ctas = ctypes.c_int(), ctypes.c_int()
+    _check(_lib.goldy_device_info(int(variant_id), ctypes.byref(sm), ctypes.byref(ctas)),
+           "goldy_device_info")
+    return sm.value, ctas.value
+
+
+def variant_id(kind: int, split: int, rc_div: int) -> int:
+    """Variant id of (kind, split-K factor, grid-cap divisor), by registry lookup."""
+    for v in range(goldy_variant_count()):
+        info = goldy_variant_info_get(v)
+        if info["kind"] == kind and info["split_k"] == split and info["rc_div"] == rc_div:
+            return v
+    raise KeyError((kind, split, rc_div))
+
+
+def kind_names() -> List[str]:
+    names = {}
+    for v in range(goldy_variant_count()):
+        info = goldy_variant_info_get(v)
+        names.setdefault(info["kind"], info["name"].split("_s")[0])
+    return [names[k] for k in sorted(names)]

@@ -1,0 +1,180 @@
+"""GPU parity: every GO-Kernel variant family against the fp64 oracle, through
+the C ABI, on seeded inputs that span several tiles and ragged tails; exact
+results on integer inputs; bit-identical results alone vs co-scheduled."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2409_02227_gb300 import goldy as G
+from paper_2409_02227_gb300 import workloads as wl
+from tests.gpu_util import Launch, check_close, check_rows, run_explicit
+
+pytestmark = pytest.mark.gpu
+
+F32, BF16 = G.GOLDY_F32, G.GOLDY_BF16
+KINDS = list(range(10))
+SWAP_KINDS = {6, 7, 8, 9}
+
+
+def vid(kind, split=1, rc=1):
+    return G.variant_id(kind, split, rc)
+
+
+def inputs(M, N, K, seed, dist="uniform", scale=1.0):
+    return (wl.random_matrix(M, K, seed, dist, scale), wl.random_matrix(K, N, seed + 1, dist, scale))
+
+
+def test_first_light_single_gemm(cuda_ok):
+    a, b = inputs(256, 256, 512, seed=0)
+    (c,) = run_explicit([a], [b], [F32], [vid(2)])
+    check_close(c, a, b, "n128_full 256x256x512")
+
+
+@pytest.mark.parametrize("out", [F32, BF16])
+@pytest.mark.parametrize("kind", KINDS)
+def test_each_kind_ragged(cuda_ok, kind, out):
+    # non-swap: M = 128 + 72 rows, N = 320 (ragged against 64/128/256 tiles), K = 7 blocks
+    # swap:     M = 40 (ragged against 32/64-row tiles), N = 296 = 2 x 128 + 40
+    M, N, K = (40, 296, 320) if kind in SWAP_KINDS else (200, 320, 448)
+    a, b = inputs(M, N, K, seed=10 + kind)
+    (c,) = run_explicit([a], [b], [out], [vid(kind)])
+    check_close(c, a, b, f"kind {kind} out {out}")
+
+
+@pytest.mark.parametrize("split", [2, 4, 8])
+@pytest.mark.parametrize("kind", [0, 3, 5, 6, 9])
+def test_split_k(cuda_ok, kind, split):
+    M, N, K = (48, 256, 1024) if kind in SWAP_KINDS else (130, 256, 1024)
+    a, b = inputs(M, N, K, seed=100 + kind * 10 + split)
+    (c,) = run_explicit([a], [b], [F32], [vid(kind, split)])
+    check_close(c, a, b, f"kind {kind} split {split}")
+    (c1,) = run_explicit([a], [b], [F32], [vid(kind, 1)])
+    # different split -> different summation order; both within the bar
+    check_close(c1, a, b, f"kind {kind} split 1")
+
+
+@pytest.mark.parametrize("kind", [0, 2, 4, 7, 8])
+def test_integer_inputs_exact(cuda_ok, kind):
+    # |a|,|b| <= 8, K <= 512: every partial sum is an integer < 2^24, exact in fp32
+    M, N, K = (64, 384, 512) if kind in SWAP_KINDS else (192, 384, 512)
+    a = wl.integer_matrix(M, K, seed=5 + kind)
+    b = wl.integer_matrix(K, N, seed=6 + kind)
+    for split in (1, 4):
+        (c,) = run_explicit([a], [b], [F32], [vid(kind, split)])
+        exact = (a.to(torch.int64) @ b.to(torch.int64)).to(torch.float32)
+        assert torch.equal(c, exact), f"kind {kind} split {split}"
+
+
+@pytest.mark.parametrize("kind", [1, 2, 7])
+def test_k_tail_and_odd_m(cuda_ok, kind):
+    M, N, K = (17, 256, 200) if kind in SWAP_KINDS else (129, 192, 200)
+    a, b = inputs(M, N, K, seed=200 + kind)
+    (c,) = run_explicit([a], [b], [F32], [vid(kind, 2)])
+    check_close(c, a, b, f"kind {kind} K tail")
+
+
+@pytest.mark.parametrize("kind", [0, 3, 6])
+def test_grid_cap_is_bit_exact(cuda_ok, kind):
+    # the resource constraint changes how many CTAs share the units, never the math
+    M, N, K = (64, 4096, 512) if kind in SWAP_KINDS else (512, 1024, 512)
+    a, b = inputs(M, N, K, seed=300 + kind)
+    outs = [run_explicit([a], [b], [F32], [vid(kind, 2, rc)])[0] for rc in (1, 2, 4)]
+    check_close(outs[0], a, b, "rc 1")
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+def test_co_schedule_invariance(cuda_ok):
+    # GEMM 0 alone vs next to three others on four streams vs after them:
+    # its bytes must not change (fixed per-element summation order)
+    shapes = [(256, 1024, 1024), (128, 1024, 4096), (32, 4096, 1024), (512, 512, 2048)]
+    vs = [vid(3, 2, 2), vid(1, 4, 4), vid(7, 2, 4), vid(5, 1, 2)]
+    outs = [F32, BF16, F32, F32]
+    A, B = zip(*[inputs(M, N, K, seed=400 + i) for i, (M, N, K) in enumerate(shapes)])
+    alone = [run_explicit([A[i]], [B[i]], [outs[i]], [vs[i]])[0] for i in range(4)]
+    conc = run_explicit(list(A), list(B), outs, vs, groups=[0, 0, 0, 0], slots=[0, 1, 2, 3])
+    seq = run_explicit(list(A), list(B), outs, vs, groups=[0, 1, 2, 3], slots=[0, 0, 0, 0])
+    mixed = run_explicit(list(A), list(B), outs, vs, groups=[0, 0, 1, 1], slots=[0, 1, 1, 0])
+    for i in range(4):
+        check_close(alone[i], A[i], B[i], f"gemm {i}")
+        for other in (conc, seq, mixed):
+            assert torch.equal(alone[i].view(torch.uint8) if alone[i].dtype == torch.bfloat16 else alone[i],
+                               other[i].view(torch.uint8) if other[i].dtype == torch.bfloat16 else other[i])
+
+
+def test_repeat_runs_reuse_workspace(cuda_ok):
+    # split-K counters must return to zero: five runs in a row give the same bytes
+    a, b = inputs(128, 1024, 4096, seed=500, dist="normal", scale=0.02)
+    s = G.goldy_schedule_build([G.desc(128, 1024, 4096, BF16)], [0], [vid(1, 8, 1)], [0])
+    L = Launch(s, [a], [b], [BF16])
+    L.run()
+    first = L.results()[0].clone()
+    check_close(first, a, b, "split 8")
+    for _ in range(4):
+        L.dC[0].fill_(float("nan"))
+        L.run()
+        assert torch.equal(L.results()[0].view(torch.int16), first.view(torch.int16))
+
+
+def test_graph_replay_matches_eager(cuda_ok):
+    shapes = [(128, 1024, 4096)] * 4
+    A, B = zip(*[inputs(M, N, K, seed=600 + i, dist="normal", scale=0.02) for i, (M, N, K) in enumerate(shapes)])
+    vs = [vid(1, 4, 4)] * 4
+    descs = [G.desc(M, N, K, BF16) for (M, N, K) in shapes]
+    s = G.goldy_schedule_build(descs, [0] * 4, vs, [0, 1, 2, 3])
+    L = Launch(s, list(A), list(B), [BF16] * 4)
+    L.run()
+    eager = [c.clone() for c in L.results()]
+    g = L.graph()
+    for c in L.dC:
+        c.fill_(float("nan"))
+    for _ in range(3):
+        G.goldy_graph_launch(g, L.streams[0].cuda_stream)
+    torch.cuda.current_stream().wait_stream(L.streams[0])
+    got = L.results()
+    for e, x in zip(eager, got):
+        assert torch.equal(e.view(torch.int16), x.view(torch.int16))
+
+
+def test_degenerate_sizes(cuda_ok):
+    a0 = torch.zeros((0, 64), dtype=torch.bfloat16)
+    b0 = wl.random_matrix(64, 128, seed=1)
+    ak = torch.zeros((70, 0), dtype=torch.bfloat16)
+    bk = torch.zeros((0, 136), dtype=torch.bfloat16)
+    a, b = inputs(33, 64, 64, seed=3)
+    descs = [G.desc(0, 128, 64), G.desc(70, 136, 0, lda=8), G.desc(33, 64, 64)]
+    s = G.goldy_schedule_build(descs, [0, 0, 0], [vid(2), vid(2), vid(6)], [0, 1, 2])
+    L = Launch(s, [a0, ak, a], [b0, bk, b], [F32, F32, F32])
+    L.run()
+    c0, ck, c = L.results()
+    assert c0.shape == (0, 128)
+    assert torch.equal(ck, torch.zeros_like(ck))
+    check_close(c, a, b, "small after degenerate")
+
+
+@pytest.mark.parametrize("name", ["pair_256", "ffn_slices", "lstm_gates"])
+def test_config_full_size(cuda_ok, name):
+    st = wl.make_config(name)
+    n = len(st.specs)
+    kinds = {"pair_256": 3, "ffn_slices": 1, "lstm_gates": 7}
+    split = {"pair_256": 1, "ffn_slices": 4, "lstm_gates": 2}
+    v = vid(kinds[name], split[name], 4)
+    outs = [s.out_dtype for s in st.specs]
+    got = run_explicit(st.a, st.b, outs, [v] * n, slots=list(range(n)))
+    for i in range(n):
+        check_close(got[i], st.a[i], st.b[i], f"{name}[{i}]")
+
+
+def test_config_hetero_pair_sampled(cuda_ok):
+    st = wl.make_config("hetero_pair")
+    vs = [vid(3, 1, 4)] * 3 + [vid(4, 1, 1)]
+    got = run_explicit(st.a, st.b, [F32] * 4, vs, slots=[0, 1, 2, 3])
+    for i in range(3):
+        check_close(got[i], st.a[i], st.b[i], f"small[{i}]")
+    rng = np.random.default_rng(3)
+    rows = np.sort(rng.choice(2048, size=48, replace=False))
+    rows[0], rows[-1] = 0, 2047
+    check_rows(got[3], st.a[3], st.b[3], rows, "big sampled rows")
+
+
+def test_device_error_word_clear(cuda_ok):
+    assert G.goldy_device_error(clear=False) == 0
