@@ -1,0 +1,549 @@
+#!/usr/bin/env python
+"""Concurrent-GEMM set benchmark on GB300.
+
+One step = one pass of the whole hot path over one synthetic GEMM set: the
+dynamic logic's plan (computed once; it is a pure function of the shapes)
+replayed as a CUDA graph of GO-Kernel launches on CD streams.  Default
+workload: the tensor-sliced Transformer FFN at low batch, 4 independent
+GEMMs of M=128, N=1024, K=4096, bf16 in, fp32 accumulate, bf16 out.
+
+Prints ONE JSON line (rank 0): TFLOP/s of the whole job (all ranks), the
+makespan, speedups over sequential and naive all-streams execution of the
+same library, cuBLAS as a reference point, a roofline entry for the dominant
+kernel, the CPU oracle as a baseline, clocks sampled during the timed region,
+and an end-to-end number through host buffers.
+
+Multi-GPU: a set of independent GEMMs needs no exchange, so N ranks run N
+independent replicas (weak scaling, no collective on the data path); the
+only collectives are the barrier and the max-reduction of the timed region.
+
+``--impl reference`` times the CPU oracle (test infrastructure) on the same
+workload instead, on the host's cores, rank 0 only.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "concurrent-GEMM set TFLOP/s and makespan speedup vs sequential and naive streams"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+CSRC = os.path.join(ROOT, "paper_2409_02227_gb300", "csrc")
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description="concurrent-GEMM set benchmark")
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=["goldy", "reference"], default="goldy")
+    ap.add_argument("--config", default="ffn_slices",
+                    choices=["pair_256", "ffn_slices", "lstm_gates", "hetero_pair"])
+    ap.add_argument("--lut", default=None, help="lookup table (default: the packaged one)")
+    ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    return ap.parse_args(argv)
+
+
+# ----------------------------------------------------------------------------- distributed
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return world, rank, local
+
+
+def dist_init(world: int, backend: str):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    if not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def reduce_max(value: float, dist, device=None) -> float:
+    """Max of `value` over ranks (the slowest rank sets the job's time)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist, device=None):
+    if dist is not None:
+        if device is not None:
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples (100 ms) around the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index                 # nvidia-smi --id: PCI bus id or index
+        self.samples = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+
+    def summary(self, t0: float, t1: float) -> dict:
+        win = [s for t, s in self.samples if t0 - 0.15 <= t <= t1 + 0.15]
+        if not win:
+            win = [s for _, s in self.samples]
+        if not win:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(s[1]) for s in win if s[1].replace(".", "").isdigit()]
+        mx = [float(s[2]) for s in win if s[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for s in win:
+            for name, v in zip(names, s[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(win)}
+
+
+# ----------------------------------------------------------------------------- helpers
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def csrc_hash() -> str:
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(CSRC)):
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(variant_name: str):
+    """DRAM bytes per launch from a committed ncu capture, if it was taken on
+    the current kernel source and the same variant; else None."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if t.get("csrc_hash") != csrc_hash() or t.get("variant") != variant_name:
+        return None
+    return t.get("dram_bytes_per_launch")
+
+
+def workload_label(specs) -> str:
+    from collections import Counter
+    c = Counter((s.M, s.N, s.K, "bf16" if s.out_dtype == 0 else "fp32") for s in specs)
+    return " + ".join(f"{n}x(M={m},N={nn},K={k},{o} out)" for (m, nn, k, o), n in c.items())
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def oracle_sample(st, budget_s: float):
+    """Run the fp64 oracle over GEMMs of the set (whole GEMMs, in order,
+    cycling) until about `budget_s` of work is done; returns
+    (flops, seconds, threads, description)."""
+    from oracle import gemm as og
+    flops = 0
+    done = []
+    t0 = time.perf_counter()
+    i = 0
+    while True:
+        og.gemm(st.a_bits(i % len(st.specs)), st.b_bits(i % len(st.specs)))
+        flops += st.specs[i % len(st.specs)].flops
+        done.append(i % len(st.specs))
+        i += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    desc = f"{len(done)} whole GEMMs of the set (indices {done[:8]}{'...' if len(done) > 8 else ''}), fp64 oracle"
+    return flops, dt, og.num_threads(), desc
+
+
+def run_reference(args, world, rank):
+    """Reference arm: the CPU oracle timed on the host's cores."""
+    if rank != 0:
+        return 0
+    from oracle import gemm as og
+    from paper_2409_02227_gb300 import workloads as wl
+    st = wl.make_config(args.config)
+    # each step computes a fixed number of output entries of every GEMM of the
+    # set (exact fp64 dot products), sized so the whole run takes about a minute
+    import numpy as np
+    K, W = max(1, args.steps), max(0, args.warmup)
+
+    def pick(i, n, step):
+        sp = st.specs[i]
+        r = np.random.default_rng([step + 1000, i])
+        return r.integers(0, sp.M, n), r.integers(0, sp.N, n)
+
+    t0 = time.perf_counter()
+    for i in range(len(st.specs)):
+        ii, jj = pick(i, 64, -1)
+        og.gemm_entries(st.a_bits(i), st.b_bits(i), ii, jj)
+    per_entry = max((time.perf_counter() - t0) / 64, 1e-7)
+    entries = int(max(1, min(4096, 60.0 / (K + W) / per_entry)))
+    flops_step = sum(2 * entries * s.K for s in st.specs)
+    for step in range(-W, K):
+        if step == 0:
+            t0 = time.perf_counter()
+        for i in range(len(st.specs)):
+            ii, jj = pick(i, entries, step)
+            og.gemm_entries(st.a_bits(i), st.b_bits(i), ii, jj)
+    dt = time.perf_counter() - t0
+    value = flops_step * K / dt / 1e12
+    sample = (f"{entries} seeded random output entries of each of the {len(st.specs)} GEMMs per step "
+              f"(exact fp64 dot products over the full K)")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": dt / K * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{args.config}: {workload_label(st.specs)}", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": og.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- GPU arm
+class SetRunner:
+    """R rotating device copies of one GEMM set, one captured graph per copy."""
+
+    def __init__(self, st, sched, copies, with_events=False):
+        import torch
+        from paper_2409_02227_gb300 import goldy as G
+        self.G = G
+        self.torch = torch
+        self.sched = sched
+        n, _, ms, ws_bytes = G.goldy_schedule_query(sched)
+        self.n = n
+        self.ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+        self.ws_bytes = ws_bytes
+        self.streams = [torch.cuda.Stream() for _ in range(max(1, ms))]
+        base_a = [a.cuda() for a in st.a]
+        base_b = [b.cuda() for b in st.b]
+        cdt = [torch.bfloat16 if s.out_dtype == 0 else torch.float32 for s in st.specs]
+        self.copies = []
+        for r in range(copies):
+            A = base_a if r == 0 else [a.clone() for a in base_a]
+            B = base_b if r == 0 else [b.clone() for b in base_b]
+            C = [torch.empty((s.M, s.N), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
+            self.copies.append((A, B, C))
+        self.events = []
+        self.graphs = []
+        torch.cuda.synchronize()
+        for A, B, C in self.copies:
+            ptrs = ([a.data_ptr() for a in A], [b.data_ptr() for b in B], [c.data_ptr() for c in C])
+            if with_events:
+                eb = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+                ee = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+                for e in eb + ee:            # torch creates the CUDA event on first record
+                    e.record()
+                torch.cuda.synchronize()
+                g = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes,
+                                            [s.cuda_stream for s in self.streams],
+                                            [e.cuda_event for e in eb], [e.cuda_event for e in ee])
+                self.events.append((eb, ee))
+            else:
+                g = G.goldy_graph_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes,
+                                         [s.cuda_stream for s in self.streams])
+            self.graphs.append(g)
+        self.main = self.streams[0]
+
+    def launch(self, k):
+        self.G.goldy_graph_launch(self.graphs[k % len(self.graphs)], self.main.cuda_stream)
+
+    def timed(self, steps):
+        torch = self.torch
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(self.main)
+        for k in range(steps):
+            self.launch(k)
+        e1.record(self.main)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    def launch_durations_ms(self):
+        out = []
+        for eb, ee in self.events:
+            for b, e in zip(eb, ee):
+                out.append(b.elapsed_time(e))
+        return out
+
+
+def cublas_reference_ms(st, copies, steps):
+    """torch.matmul (cuBLAS) for the same set, back to back on one stream,
+    captured in a CUDA graph per rotating copy: a reference point only."""
+    import torch
+    base_a = [a.cuda() for a in st.a]
+    base_b = [b.cuda() for b in st.b]
+    graphs = []
+    outs = []
+    s = torch.cuda.Stream()
+    for r in range(copies):
+        A = base_a if r == 0 else [a.clone() for a in base_a]
+        B = base_b if r == 0 else [b.clone() for b in base_b]
+        with torch.cuda.stream(s):
+            for a, b in zip(A, B):
+                torch.matmul(a, b)          # warm cuBLAS handles outside the capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            o = [torch.matmul(a, b) for a, b in zip(A, B)]
+        graphs.append(g)
+        outs.append(o)
+    for k in range(10):
+        graphs[k % copies].replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for k in range(steps):
+        graphs[k % copies].replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def e2e_measure(st, sched, steps):
+    """Same metric through host buffers: each step copies A, B from pinned
+    host memory, runs the schedule, and reads C back to pinned host memory."""
+    import torch
+    from paper_2409_02227_gb300 import goldy as G
+    _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
+    streams = [torch.cuda.Stream() for _ in range(max(1, ms))]
+    ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+    hA = [a.pin_memory() for a in st.a]
+    hB = [b.pin_memory() for b in st.b]
+    cdt = [torch.bfloat16 if s.out_dtype == 0 else torch.float32 for s in st.specs]
+    hC = [torch.empty((s.M, s.N), dtype=d).pin_memory() for s, d in zip(st.specs, cdt)]
+    dA = [torch.empty_like(a, device="cuda") for a in st.a]
+    dB = [torch.empty_like(b, device="cuda") for b in st.b]
+    dC = [torch.empty((s.M, s.N), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
+    main = streams[0]
+    A = [a.data_ptr() for a in dA]
+    B = [b.data_ptr() for b in dB]
+    C = [c.data_ptr() for c in dC]
+    sp = [s.cuda_stream for s in streams]
+
+    def step():
+        with torch.cuda.stream(main):
+            for d, h in zip(dA + dB, hA + hB):
+                d.copy_(h, non_blocking=True)
+        G.goldy_run(sched, A, B, C, ws.data_ptr(), ws_bytes, sp)
+        with torch.cuda.stream(main):
+            for h, d in zip(hC, dC):
+                h.copy_(d, non_blocking=True)
+
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(main)
+    for _ in range(steps):
+        step()
+    e1.record(main)
+    torch.cuda.synchronize()
+    ms_step = e0.elapsed_time(e1) / steps
+    h2d = sum(a.numel() * a.element_size() for a in hA + hB)
+    d2h = sum(c.numel() * c.element_size() for c in hC)
+    return ms_step, h2d, d2h
+
+
+def run_gpu(args, world, rank, local):
+    import torch
+    dist = dist_init(world, "nccl")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    from paper_2409_02227_gb300 import goldy as G
+    from paper_2409_02227_gb300 import workloads as wl
+
+    st = wl.make_config(args.config)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO)
+    plan = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
+    props = torch.cuda.get_device_properties(device)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 1024 * 1024))
+    in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
+    copies = max(2, math.ceil(2 * l2 / in_bytes))
+
+    runner = SetRunner(st, sched, copies, with_events=True)
+    for k in range(max(3, args.warmup)):
+        runner.launch(k)
+    torch.cuda.synchronize()
+
+    try:
+        gpu_id = "%08X:%02X:%02X.0" % (props.pci_domain_id, props.pci_bus_id, props.pci_device_id)
+    except AttributeError:
+        gpu_id = str(local)
+    sampler = ClockSampler(gpu_id)
+    sampler.start()
+    time.sleep(0.25)
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    elapsed_ms = runner.timed(args.steps)
+    t_wall1 = time.time()
+    barrier(dist, device)
+    sampler.stop()
+    elapsed_ms = reduce_max(elapsed_ms, dist, device)
+    if G.goldy_device_error(clear=True) != 0:
+        raise RuntimeError("a GO-Kernel reported a bounded-wait timeout during the timed region")
+    ms_step = elapsed_ms / args.steps
+    value = world * st.flops / (ms_step * 1e-3) / 1e12
+
+    # dominant kernel: the variant carrying the most FLOPs in the plan
+    by_variant = {}
+    for i, (g, v, slot, cd) in enumerate(plan):
+        by_variant.setdefault(v, []).append(i)
+    dom_v = max(by_variant, key=lambda v: sum(st.specs[i].flops for i in by_variant[v]))
+    dom_idx = by_variant[dom_v]
+    durs = []
+    for eb, ee in runner.events:
+        for i in dom_idx:
+            durs.append(eb[i].elapsed_time(ee[i]))
+    dur_ms = statistics.mean(durs)
+    bytes_per_launch = statistics.mean(st.specs[i].bytes for i in dom_idx)
+    flops_per_launch = statistics.mean(st.specs[i].flops for i in dom_idx)
+    hbm, tf_burst, tf_sust, peak_src = peaks()
+    ai = flops_per_launch / bytes_per_launch
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    vname = G.goldy_variant_info_get(dom_v)["name"]
+    if ai < ridge:
+        achieved = bytes_per_launch / (dur_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm}
+    else:
+        achieved = flops_per_launch / (dur_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": achieved / tf_burst}
+    roof["traffic"] = recorded_traffic(vname)
+    roof.update({"kernel": vname, "launch_us": dur_ms * 1e3, "launches_sampled": len(durs),
+                 "per_launch": {"algorithmic_bytes": bytes_per_launch, "flops": flops_per_launch},
+                 "peak_source": f"{peak_src} ({'HBM copy' if roof['bound'] == 'hbm' else 'cuBLAS bf16 burst'})"})
+
+    set_roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
+    launches_per_step = sum(1 for s in st.specs if s.M and s.N)
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{args.config}: {workload_label(st.specs)}",
+                   "l2": f"inputs larger than L2: {copies} rotating device copies of the set "
+                         f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2)",
+                   "launch": "CUDA graph replay of the planned schedule",
+                   "plan": [{"gemm": i, "group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl,
+                             "cd": cd} for i, (g, v, sl, cd) in enumerate(plan)],
+                   "parallelism": f"replicas x{world}"},
+        "makespan_us": ms_step * 1e3,
+        "set_roof_us": set_roof_us,
+        "set_roofline_frac": set_roof_us / (ms_step * 1e3),
+        "gpu_launches": launches_per_step * args.steps,
+        "roofline": roof,
+    }
+    clocks = sampler.summary(t_wall0, t_wall1)
+    line["clocks"] = clocks
+
+    if not args.no_compare:
+        csteps = max(200, min(args.steps, 5000))
+        comp = {}
+        for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
+                            ("go_all_concurrent", G.GOLDY_PLAN_GO)):
+            s2 = G.goldy_plan(descs, lut, flags)
+            r2 = SetRunner(st, s2, copies)
+            for k in range(10):
+                r2.launch(k)
+            torch.cuda.synchronize()
+            comp[name] = r2.timed(csteps) / csteps * 1e3
+            del r2
+        auto_us = SetRunner(st, sched, copies)
+        for k in range(10):
+            auto_us.launch(k)
+        torch.cuda.synchronize()
+        a_us = auto_us.timed(csteps) / csteps * 1e3
+        del auto_us
+        cb = cublas_reference_ms(st, copies, csteps) * 1e3
+        line["comparisons_us"] = {"goldyloc": a_us, **comp, "cublas_sequential_reference": cb}
+        line["speedup_vs_sequential"] = comp["sequential"] / a_us
+        line["speedup_vs_naive_streams"] = comp["naive_streams"] / a_us
+
+    e2e_steps = max(5, min(args.steps, 200))
+    e_ms, h2d, d2h = e2e_measure(st, sched, e2e_steps)
+    e_ms = reduce_max(e_ms, dist, device)
+    line["e2e"] = {"value": world * st.flops / (e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                   "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
+                   "steps": e2e_steps}
+
+    if rank == 0 and not args.no_cpu:
+        flops, secs, threads, desc = oracle_sample(st, budget_s=10.0)
+        line["cpu_baseline"] = {"value": flops / secs / 1e12, "unit": "TFLOP/s", "cores": threads,
+                                "kind": "oracle", "sample": desc + f", {secs:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier(device_ids=[local])
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+    return run_gpu(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -196,6 +196,21 @@ goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void
                        void* const* C, void* workspace, size_t workspace_bytes,
                        void* const* streams, int n_streams);
 
+/* Options of goldy_run_ex / goldy_graph_create_ex (all fields may be null).
+ * ev_begin[i] / ev_end[i] (cudaEvent_t as void*, caller-created, one pair per
+ * GEMM) are recorded on GEMM i's stream right before and right after its
+ * kernel launch, so the caller can time each launch on the stream it runs on.
+ * Inside a graph capture they become event-record nodes of the graph. */
+typedef struct goldy_run_opts {
+  void* const* ev_begin;
+  void* const* ev_end;
+} goldy_run_opts;
+
+/* goldy_run with options; opts may be null (then identical to goldy_run). */
+goldy_status goldy_run_ex(const goldy_schedule* s, const void* const* A, const void* const* B,
+                          void* const* C, void* workspace, size_t workspace_bytes,
+                          void* const* streams, int n_streams, const goldy_run_opts* opts);
+
 /* Capture goldy_run(...) with these exact pointers into a CUDA graph, for
  * replay with one launch (the closest host-side analogue of the command
  * processor dispatching a whole set).  The streams must be idle.  The graph
@@ -204,6 +219,11 @@ goldy_status goldy_graph_create(const goldy_schedule* s, const void* const* A,
                                 const void* const* B, void* const* C, void* workspace,
                                 size_t workspace_bytes, void* const* streams, int n_streams,
                                 goldy_graph** out);
+/* goldy_graph_create with run options (event hooks captured into the graph). */
+goldy_status goldy_graph_create_ex(const goldy_schedule* s, const void* const* A,
+                                   const void* const* B, void* const* C, void* workspace,
+                                   size_t workspace_bytes, void* const* streams, int n_streams,
+                                   const goldy_run_opts* opts, goldy_graph** out);
 /* Launch a captured graph on `stream` (asynchronous). */
 goldy_status goldy_graph_launch(const goldy_graph* g, void* stream);
 void goldy_graph_free(goldy_graph* g);

@@ -198,9 +198,28 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
 
 using namespace goldy;
 
+namespace {
+// Record a caller's timing event on `stream`; inside a capture it must be an
+// external record to become a real node of the graph.
+cudaError_t record_hook(void* ev, cudaStream_t stream) {
+  if (!ev) return cudaSuccess;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(stream, &cs);
+  if (e != cudaSuccess) return e;
+  return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev), stream,
+                                  cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : 0);
+}
+}  // namespace
+
 extern "C" goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void* const* B,
                                   void* const* C, void* workspace, size_t workspace_bytes, void* const* streams,
                                   int n_streams) {
+  return goldy_run_ex(s, A, B, C, workspace, workspace_bytes, streams, n_streams, nullptr);
+}
+
+extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                     void* const* C, void* workspace, size_t workspace_bytes, void* const* streams,
+                                     int n_streams, const goldy_run_opts* opts) {
   if (!s || !A || !B || !C || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
   if (n_streams < s->max_streams) return fail(GOLDY_ERR_INVALID_ARG, "fewer streams than the schedule needs");
   if (s->workspace_bytes > 0) {
@@ -259,8 +278,17 @@ extern "C" goldy_status goldy_run(const goldy_schedule* s, const void* const* A,
     }
     for (int i : grp.members) {
       const GemmPlan& gp = s->gemms[i];
-      st = launch_gemm(*d, gp, A[i], B[i], C[i], ws, static_cast<cudaStream_t>(streams[gp.slot]));
+      cudaStream_t st_i = static_cast<cudaStream_t>(streams[gp.slot]);
+      if (opts && opts->ev_begin) {
+        cudaError_t e = record_hook(opts->ev_begin[i], st_i);
+        if (e != cudaSuccess) return cuda_fail(e, "timing event");
+      }
+      st = launch_gemm(*d, gp, A[i], B[i], C[i], ws, st_i);
       if (st != GOLDY_OK) return st;
+      if (opts && opts->ev_end) {
+        cudaError_t e = record_hook(opts->ev_end[i], st_i);
+        if (e != cudaSuccess) return cuda_fail(e, "timing event");
+      }
     }
     if (side) {
       for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
@@ -282,12 +310,19 @@ struct goldy_graph {
 extern "C" goldy_status goldy_graph_create(const goldy_schedule* s, const void* const* A, const void* const* B,
                                            void* const* C, void* workspace, size_t workspace_bytes,
                                            void* const* streams, int n_streams, goldy_graph** out) {
+  return goldy_graph_create_ex(s, A, B, C, workspace, workspace_bytes, streams, n_streams, nullptr, out);
+}
+
+extern "C" goldy_status goldy_graph_create_ex(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                              void* const* C, void* workspace, size_t workspace_bytes,
+                                              void* const* streams, int n_streams, const goldy_run_opts* opts,
+                                              goldy_graph** out) {
   if (!out || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
   *out = nullptr;
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   cudaError_t e = cudaStreamBeginCapture(main, cudaStreamCaptureModeThreadLocal);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamBeginCapture");
-  goldy_status st = goldy_run(s, A, B, C, workspace, workspace_bytes, streams, n_streams);
+  goldy_status st = goldy_run_ex(s, A, B, C, workspace, workspace_bytes, streams, n_streams, opts);
   std::string why = st == GOLDY_OK ? "" : goldy_last_error();
   cudaGraph_t graph = nullptr;
   e = cudaStreamEndCapture(main, &graph);

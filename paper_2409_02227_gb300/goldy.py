@@ -56,6 +56,10 @@ class goldy_gemm_desc(ctypes.Structure):
                 ("c_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class goldy_run_opts(ctypes.Structure):
+    _fields_ = [("ev_begin", ctypes.POINTER(ctypes.c_void_p)), ("ev_end", ctypes.POINTER(ctypes.c_void_p))]
+
+
 class goldy_variant_info(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("id", "kind", "mma_m", "mma_n", "swap_ab", "stages", "acc_stages", "tmem_cols",
@@ -93,6 +97,8 @@ def _load():
         "goldy_schedule_free": ([P], None),
         "goldy_run": ([P, PP, PP, PP, P, SZ, PP, I], I),
         "goldy_graph_create": ([P, PP, PP, PP, P, SZ, PP, I, PP], I),
+        "goldy_run_ex": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts)], I),
+        "goldy_graph_create_ex": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts), PP], I),
         "goldy_graph_launch": ([P, P], I),
         "goldy_graph_free": ([P], None),
         "goldy_device_error": ([IP, I], I),
@@ -255,6 +261,42 @@ def goldy_graph_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Seque
     _check(_lib.goldy_graph_create(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                                    int(workspace_bytes), _ptrs(streams), len(streams),
                                    ctypes.byref(out)), "goldy_graph_create")
+    return Graph(out)
+
+
+def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]]):
+    o = goldy_run_opts()
+    keep = []
+    if ev_begin is not None:
+        arr = _ptrs(ev_begin)
+        keep.append(arr)
+        o.ev_begin = ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))
+    if ev_end is not None:
+        arr = _ptrs(ev_end)
+        keep.append(arr)
+        o.ev_end = ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))
+    return o, keep
+
+
+def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
+                 workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
+                 ev_end: Optional[Sequence[int]] = None) -> None:
+    """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints)."""
+    o, _keep = _opts(ev_begin, ev_end)
+    _check(_lib.goldy_run_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
+                             int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o)),
+           "goldy_run_ex")
+
+
+def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int],
+                          workspace: int, workspace_bytes: int, streams: Sequence[int],
+                          ev_begin: Optional[Sequence[int]] = None,
+                          ev_end: Optional[Sequence[int]] = None) -> Graph:
+    o, _keep = _opts(ev_begin, ev_end)
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_graph_create_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
+                                      int(workspace_bytes), _ptrs(streams), len(streams),
+                                      ctypes.byref(o), ctypes.byref(out)), "goldy_graph_create_ex")
     return Graph(out)
 
 

@@ -1,0 +1,76 @@
+"""Host-side logic that needs no GPU: the profiler's preferred-CD rule and LUT
+writer against the oracle's independent versions, and bench.py's multi-rank
+aggregation (barrier + max over ranks) on world_size-2 gloo process groups."""
+import os
+import random
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+from oracle import planner_ref as pr
+from paper_2409_02227_gb300 import goldy as G
+from paper_2409_02227_gb300 import profile_lut as P
+
+
+def test_preferred_cd_matches_oracle():
+    rng = random.Random(5)
+    for _ in range(5000):
+        sp = {1: 1.0}
+        for cd in (2, 4, 8, 16):
+            if rng.random() < 0.9:
+                sp[cd] = rng.choice([rng.uniform(0.5, 2.5), rng.uniform(0.98, 1.08)])
+        assert P.preferred_cd(sp) == pr.preferred_cd(sp), sp
+
+
+def test_lut_writer_matches_oracle_format():
+    rng = random.Random(9)
+    keys = {(rng.randint(3, 13), rng.randint(7, 14), rng.randint(7, 14), rng.randint(0, 1)) for _ in range(50)}
+    entries = [(k, rng.choice(pr.CD_CLASSES), [rng.randrange(120) for _ in range(5)]) for k in keys]
+    mine = P.write_lut(entries, 120, 152)
+    ref = pr.write_lut([pr.Entry(k, p, tuple(v)) for k, p, v in entries], 120, 152)
+    assert mine == ref
+    G.goldy_lut_from_memory(mine)
+
+
+def test_bucket_shapes_and_candidates():
+    assert P.bucket_shape((7, 10, 12, 0)) == (128, 1024, 4096, 0)
+    c = P.candidates(32, 4096, 1024, 152)
+    kinds = {k for k, _ in c}
+    assert {6, 7, 8, 9} <= kinds                      # transposed tiles offered for skinny M
+    assert all(s in (1, 2, 4, 8) for _, s in c)
+    assert not {6, 7, 8, 9} & {k for k, _ in P.candidates(512, 1024, 1024, 152)}
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    import bench
+    w, r, l = bench.dist_env()
+    dist = bench.dist_init(w, "gloo")
+    bench.barrier(dist)
+    got = bench.reduce_max(10.0 + rank, dist)
+    q.put((r, got))
+    dist.destroy_process_group()
+
+
+def test_multi_rank_max_over_gloo():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = dict(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    assert res == {0: 11.0, 1: 11.0}
