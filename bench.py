@@ -302,6 +302,10 @@ class SetRunner:
             self.graphs.append(g)
         self.main = self.streams[0]
 
+    def __del__(self):
+        # destroy the graphs before the buffers they read and write
+        self.graphs.clear()
+
     def launch(self, k):
         self.G.goldy_graph_launch(self.graphs[k % len(self.graphs)], self.main.cuda_stream)
 
@@ -331,10 +335,12 @@ def cublas_reference_ms(st, copies, steps):
     base_b = [b.cuda() for b in st.b]
     graphs = []
     outs = []
+    keep = []                   # every captured graph reads its own inputs: keep them all alive
     s = torch.cuda.Stream()
     for r in range(copies):
         A = base_a if r == 0 else [a.clone() for a in base_a]
         B = base_b if r == 0 else [b.clone() for b in base_b]
+        keep.append((A, B))
         with torch.cuda.stream(s):
             for a, b in zip(A, B):
                 torch.matmul(a, b)          # warm cuBLAS handles outside the capture
@@ -353,7 +359,9 @@ def cublas_reference_ms(st, copies, steps):
         graphs[k % copies].replay()
     e1.record()
     torch.cuda.synchronize()
-    return e0.elapsed_time(e1) / steps
+    ms = e0.elapsed_time(e1) / steps
+    del graphs, outs, keep
+    return ms
 
 
 def e2e_measure(st, sched, steps):
