@@ -1,7 +1,8 @@
 """Build ``libgoldy.so`` (the C-ABI library) in-tree for sm_103a.
 
 Plain nvcc/g++ invocations, one object per translation unit, compiled in
-parallel: ``planner.cpp`` (host C++), ``runtime.cu`` (launch manager) and
+parallel: ``planner.cpp`` (host C++), ``runtime.cu`` (launch manager),
+``noalloc.cu`` (the entry point with a compiled-in scratch array) and
 ``kernels.cu`` once per GO-Kernel kind (``-DGOLDY_KIND=k``).  Objects go to
 ``_build/`` next to this file and the library to
 ``paper_2409_02227_gb300/libgoldy.so``; both are git-ignored.  A rebuild is
@@ -50,6 +51,7 @@ def _jobs(ptxas_verbose: bool):
     jobs.append(("planner", ["g++", "-std=c++17", "-O2", "-fPIC", "-Wall", "-I", CSRC, "-I", INCLUDE,
                              "-c", os.path.join(CSRC, "planner.cpp")]))
     jobs.append(("runtime", cu + ["-c", os.path.join(CSRC, "runtime.cu")]))
+    jobs.append(("noalloc", cu + ["-c", os.path.join(CSRC, "noalloc.cu")]))
     for k in range(NUM_KINDS):
         jobs.append((f"kernels_k{k}", cu + [f"-DGOLDY_KIND={k}", "-c", os.path.join(CSRC, "kernels.cu")]))
     return jobs

@@ -386,3 +386,16 @@ extern "C" goldy_status goldy_device_info(int variant_id, int* sm_count, int* ct
   if (ctas_per_sm) *ctas_per_sm = ctas;
   return ok();
 }
+
+namespace goldy {
+// Launch one GEMM whose plan fields (kind, tiles, split, workspace offsets)
+// are already filled in, with `ws` as the workspace base.  Shares the
+// per-device setup and the launch code of goldy_run.
+goldy_status launch_planned_gemm(const GemmPlan& gp, const void* A, const void* B, void* C, unsigned char* ws,
+                                 void* stream) {
+  DeviceState* d = nullptr;
+  goldy_status st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+  return launch_gemm(*d, gp, A, B, C, ws, static_cast<cudaStream_t>(stream));
+}
+}  // namespace goldy

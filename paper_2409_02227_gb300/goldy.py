@@ -101,6 +101,7 @@ def _load():
         "goldy_graph_create_ex": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts), PP], I),
         "goldy_graph_launch": ([P, P], I),
         "goldy_graph_free": ([P], None),
+        "goldy_gemm_noalloc": ([DP, I, P, P, P, P], I),
         "goldy_device_error": ([IP, I], I),
         "goldy_device_info": ([I, IP, IP], I),
     }
@@ -302,6 +303,13 @@ def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Se
 
 def goldy_graph_launch(g: Graph, stream: int) -> None:
     _check(_lib.goldy_graph_launch(g.ptr, int(stream) or None), "goldy_graph_launch")
+
+
+def goldy_gemm_noalloc(d: goldy_gemm_desc, variant: int, A: int, B: int, C: int, stream: int = 0) -> None:
+    """One GEMM with the library's compiled-in split-K scratch (no device
+    allocation anywhere); see goldy.h for who needs it and its limits."""
+    _check(_lib.goldy_gemm_noalloc(ctypes.byref(d), int(variant), int(A) or None, int(B) or None,
+                                   int(C) or None, int(stream) or None), "goldy_gemm_noalloc")
 
 
 def goldy_device_error(clear: bool = True) -> int:
