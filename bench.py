@@ -52,6 +52,8 @@ def parse_args(argv=None):
     ap.add_argument("--config", default="ffn_slices",
                     choices=["pair_256", "ffn_slices", "lstm_gates", "hetero_pair"])
     ap.add_argument("--lut", default=None, help="lookup table (default: the packaged one)")
+    ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
+                    help="fused: a wave's same-kind GEMMs share one launch; streams: one launch per GEMM")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     return ap.parse_args(argv)
@@ -309,15 +311,27 @@ class SetRunner:
     def launch(self, k):
         self.G.goldy_graph_launch(self.graphs[k % len(self.graphs)], self.main.cuda_stream)
 
-    def timed(self, steps):
+    def timed(self, steps, step_events=0):
+        """Elapsed ms of `steps` back-to-back replays; with `step_events`, the
+        last that many replays are also bracketed by their own event pair on
+        the launching stream (returned as a list of ms)."""
         torch = self.torch
+        step_events = min(step_events, steps)
+        pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in range(step_events)]
+        first = steps - step_events
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(self.main)
         for k in range(steps):
-            self.launch(k)
+            if k >= first:
+                pairs[k - first][0].record(self.main)
+                self.launch(k)
+                pairs[k - first][1].record(self.main)
+            else:
+                self.launch(k)
         e1.record(self.main)
         torch.cuda.synchronize()
-        return e0.elapsed_time(e1)
+        return e0.elapsed_time(e1), [a.elapsed_time(b) for a, b in pairs]
 
     def launch_durations_ms(self):
         out = []
@@ -420,14 +434,18 @@ def run_gpu(args, world, rank, local):
     st = wl.make_config(args.config)
     descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
     lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
-    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO)
+    launch_flag = G.GOLDY_PLAN_FUSED if args.launch == "fused" else 0
+    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | launch_flag)
     plan = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
+    kinds = {(G.goldy_variant_info_get(v)["kind"], st.specs[i].out_dtype) for i, (_, v, _, _) in enumerate(plan)}
+    n_groups = G.goldy_schedule_query(sched)[1]
+    single_launch = bool(launch_flag) and n_groups == 1 and len(kinds) == 1 and plan[0][3] >= len(descs)
     props = torch.cuda.get_device_properties(device)
     l2 = int(getattr(props, "L2_cache_size", 126 * 1024 * 1024))
     in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
     copies = max(2, math.ceil(2 * l2 / in_bytes))
 
-    runner = SetRunner(st, sched, copies, with_events=True)
+    runner = SetRunner(st, sched, copies)
     for k in range(max(3, args.warmup)):
         runner.launch(k)
     torch.cuda.synchronize()
@@ -442,7 +460,7 @@ def run_gpu(args, world, rank, local):
     barrier(dist, device)
     torch.cuda.synchronize()
     t_wall0 = time.time()
-    elapsed_ms = runner.timed(args.steps)
+    elapsed_ms, step_ms = runner.timed(args.steps, step_events=64 if single_launch else 0)
     t_wall1 = time.time()
     barrier(dist, device)
     sampler.stop()
@@ -458,17 +476,27 @@ def run_gpu(args, world, rank, local):
         by_variant.setdefault(v, []).append(i)
     dom_v = max(by_variant, key=lambda v: sum(st.specs[i].flops for i in by_variant[v]))
     dom_idx = by_variant[dom_v]
-    durs = []
-    for eb, ee in runner.events:
-        for i in dom_idx:
-            durs.append(eb[i].elapsed_time(ee[i]))
+    if single_launch:
+        # one launch per step: the events around each of the last 64 timed
+        # replays on the launching stream time that launch; it covers all GEMMs
+        durs = step_ms
+        dom_idx = list(range(len(descs)))
+        timing_note = "events around the single fused launch of each of the last 64 timed steps"
+    else:
+        inst = SetRunner(st, sched, copies, with_events=True)
+        for k in range(2 * copies):
+            inst.launch(k)
+        torch.cuda.synchronize()
+        durs = [eb[i].elapsed_time(ee[i]) for eb, ee in inst.events for i in dom_idx]
+        del inst
+        timing_note = "events recorded around each launch on its own stream inside an instrumented copy of the graph"
     dur_ms = statistics.mean(durs)
-    bytes_per_launch = statistics.mean(st.specs[i].bytes for i in dom_idx)
-    flops_per_launch = statistics.mean(st.specs[i].flops for i in dom_idx)
+    bytes_per_launch = sum(st.specs[i].bytes for i in dom_idx) / (1 if single_launch else len(dom_idx))
+    flops_per_launch = sum(st.specs[i].flops for i in dom_idx) / (1 if single_launch else len(dom_idx))
     hbm, tf_burst, tf_sust, peak_src = peaks()
     ai = flops_per_launch / bytes_per_launch
     ridge = tf_burst * 1e12 / (hbm * 1e9)
-    vname = G.goldy_variant_info_get(dom_v)["name"]
+    vname = G.goldy_variant_info_get(dom_v)["name"] + (f" fused x{len(descs)}" if single_launch else "")
     if ai < ridge:
         achieved = bytes_per_launch / (dur_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm}
@@ -478,11 +506,12 @@ def run_gpu(args, world, rank, local):
                 "frac": achieved / tf_burst}
     roof["traffic"] = recorded_traffic(vname)
     roof.update({"kernel": vname, "launch_us": dur_ms * 1e3, "launches_sampled": len(durs),
+                 "timing": timing_note,
                  "per_launch": {"algorithmic_bytes": bytes_per_launch, "flops": flops_per_launch},
                  "peak_source": f"{peak_src} ({'HBM copy' if roof['bound'] == 'hbm' else 'cuBLAS bf16 burst'})"})
 
     set_roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
-    launches_per_step = sum(1 for s in st.specs if s.M and s.N)
+    launches_per_step = 1 if single_launch else sum(1 for s in st.specs if s.M and s.N and s.K)
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
@@ -490,7 +519,7 @@ def run_gpu(args, world, rank, local):
         "config": {"workload": f"{args.config}: {workload_label(st.specs)}",
                    "l2": f"inputs larger than L2: {copies} rotating device copies of the set "
                          f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2)",
-                   "launch": "CUDA graph replay of the planned schedule",
+                   "launch": f"CUDA graph replay of the planned schedule ({args.launch} launch mode)",
                    "plan": [{"gemm": i, "group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl,
                              "cd": cd} for i, (g, v, sl, cd) in enumerate(plan)],
                    "parallelism": f"replicas x{world}"},
@@ -507,22 +536,19 @@ def run_gpu(args, world, rank, local):
         csteps = max(200, min(args.steps, 5000))
         comp = {}
         for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
-                            ("go_all_concurrent", G.GOLDY_PLAN_GO)):
+                            ("go_all_concurrent", G.GOLDY_PLAN_GO),
+                            ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
+                            ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
             s2 = G.goldy_plan(descs, lut, flags)
             r2 = SetRunner(st, s2, copies)
             for k in range(10):
                 r2.launch(k)
             torch.cuda.synchronize()
-            comp[name] = r2.timed(csteps) / csteps * 1e3
+            comp[name] = r2.timed(csteps)[0] / csteps * 1e3
             del r2
-        auto_us = SetRunner(st, sched, copies)
-        for k in range(10):
-            auto_us.launch(k)
-        torch.cuda.synchronize()
-        a_us = auto_us.timed(csteps) / csteps * 1e3
-        del auto_us
+        a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
         cb = cublas_reference_ms(st, copies, csteps) * 1e3
-        line["comparisons_us"] = {"goldyloc": a_us, **comp, "cublas_sequential_reference": cb}
+        line["comparisons_us"] = {**comp, "cublas_sequential_reference": cb}
         line["speedup_vs_sequential"] = comp["sequential"] / a_us
         line["speedup_vs_naive_streams"] = comp["naive_streams"] / a_us
 

@@ -86,6 +86,13 @@ typedef struct goldy_graph goldy_graph;
 #define GOLDY_PLAN_DEFAULT 2
 #define GOLDY_PLAN_GO 3
 #define GOLDY_PLAN_FORCE_CD 4
+/* Launch-mode bit, combinable with any policy above.  FUSED: within each
+ * group, the GEMMs that run at the same time (a "wave" of CD members) and
+ * share a kernel kind and output dtype go into ONE persistent launch over the
+ * concatenation of their tiles (at most 16 GEMMs per launch); its grid cap is
+ * the sum of the members' caps.  Without it every GEMM is its own launch on
+ * its slot's stream.  The plan (groups, CDs, variants, slots) is the same. */
+#define GOLDY_PLAN_FUSED 0x10
 
 #define GOLDY_MAX_GEMMS 64      /* GEMMs per plan */
 #define GOLDY_MAX_STREAMS 16    /* concurrency degrees 1, 2, 4, 8, 16 (Sec. 4.3) */
@@ -155,9 +162,10 @@ goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const goldy_lut* lu
  * chosen schedule): GEMM i runs in group group_of[i] (groups are run in
  * increasing order, ids 0 .. n_groups-1 all used), with variant
  * variant_of[i], on stream slot slot_of[i] (< GOLDY_MAX_STREAMS).  A group's
- * CD is its number of distinct slots. */
+ * CD is its number of distinct slots.  flags: 0 or GOLDY_PLAN_FUSED (waves are
+ * then the group's members taken CD at a time, in GEMM index order). */
 goldy_status goldy_schedule_build(const goldy_gemm_desc* descs, int n, const int* group_of,
-                                  const int* variant_of, const int* slot_of,
+                                  const int* variant_of, const int* slot_of, int flags,
                                   goldy_schedule** out);
 
 /* Sizes of a schedule.  workspace_bytes is the device workspace goldy_run

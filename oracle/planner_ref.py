@@ -64,6 +64,7 @@ POLICY_SEQUENTIAL = 1
 POLICY_DEFAULT = 2
 POLICY_GO = 3
 POLICY_FORCE_CD = 4
+FUSED = 0x10            # launch-mode bit: does not change the plan, only how it is launched
 
 DTYPE_BF16 = 0
 DTYPE_F32 = 1
@@ -170,7 +171,7 @@ def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
         raise PlanError("bad count")
     policy = flags & 0xF
     forced = (flags >> 8) & 0xFF
-    if (flags & ~0xFF0F) or policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
+    if (flags & ~0xFF1F) or policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
         raise PlanError("bad flags")
     keys = [bucket_key(d.M, d.N, d.K, d.out_dtype) for d in descs]
     ents = [lookup(entries, k) for k in keys]

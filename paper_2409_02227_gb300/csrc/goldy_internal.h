@@ -110,18 +110,20 @@ struct Group {
 
 struct Runtime;              // CUDA-side state (events), defined in runtime.cu
 
-// Host stubs of the GO-Kernel of each kind, for fp32 (0) or bf16 (1) output;
-// kernels.cu is compiled once per kind (-DGOLDY_KIND=k) to define them.
-const void* kernel_fn_k0(int out_bf16);
-const void* kernel_fn_k1(int out_bf16);
-const void* kernel_fn_k2(int out_bf16);
-const void* kernel_fn_k3(int out_bf16);
-const void* kernel_fn_k4(int out_bf16);
-const void* kernel_fn_k5(int out_bf16);
-const void* kernel_fn_k6(int out_bf16);
-const void* kernel_fn_k7(int out_bf16);
-const void* kernel_fn_k8(int out_bf16);
-const void* kernel_fn_k9(int out_bf16);
+// Host stubs of the GO-Kernel of each kind, for fp32 (0) or bf16 (1) output,
+// one GEMM per launch (fused = 0) or up to kMaxFused (fused = 1); kernels.cu
+// is compiled once per kind (-DGOLDY_KIND=k) to define them.
+constexpr int kMaxFused = 16;
+const void* kernel_fn_k0(int out_bf16, int fused);
+const void* kernel_fn_k1(int out_bf16, int fused);
+const void* kernel_fn_k2(int out_bf16, int fused);
+const void* kernel_fn_k3(int out_bf16, int fused);
+const void* kernel_fn_k4(int out_bf16, int fused);
+const void* kernel_fn_k5(int out_bf16, int fused);
+const void* kernel_fn_k6(int out_bf16, int fused);
+const void* kernel_fn_k7(int out_bf16, int fused);
+const void* kernel_fn_k8(int out_bf16, int fused);
+const void* kernel_fn_k9(int out_bf16, int fused);
 
 }  // namespace goldy
 

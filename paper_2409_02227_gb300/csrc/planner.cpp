@@ -243,7 +243,7 @@ extern "C" goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const go
   if (!lut) return fail(GOLDY_ERR_LUT, "no lookup table");
   const int policy = flags & 0xF;
   const int forced = (flags >> 8) & 0xFF;
-  if ((flags & ~0xFF0F) != 0 || policy > GOLDY_PLAN_FORCE_CD ||
+  if ((flags & ~0xFF1F) != 0 || policy > GOLDY_PLAN_FORCE_CD ||
       (policy == GOLDY_PLAN_FORCE_CD && forced < 1))
     return fail(GOLDY_ERR_INVALID_ARG, "bad flags");
   goldy_schedule* s = nullptr;
@@ -347,12 +347,14 @@ extern "C" goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const go
 }
 
 extern "C" goldy_status goldy_schedule_build(const goldy_gemm_desc* descs, int n, const int* group_of,
-                                             const int* variant_of, const int* slot_of,
+                                             const int* variant_of, const int* slot_of, int flags,
                                              goldy_schedule** out) {
   if (!group_of || !variant_of || !slot_of) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  if ((flags & ~GOLDY_PLAN_FUSED) != 0) return fail(GOLDY_ERR_INVALID_ARG, "bad flags");
   goldy_schedule* s = nullptr;
   goldy_status st = new_schedule(descs, n, &s);
   if (st != GOLDY_OK) return st;
+  s->flags = flags;
   int n_groups = 0;
   for (int i = 0; i < n; ++i) {
     if (group_of[i] < 0 || group_of[i] >= n || variant_of[i] < 0 || variant_of[i] >= kNumVariants ||

@@ -5,8 +5,10 @@
 // (Sec. 4.4).  Here each group of the schedule forks from streams[0] with an
 // event, launches its GEMMs round-robin onto the group's stream slots (so at
 // most CD GEMMs are in flight, each stream running its GEMMs back to back),
-// and joins back into streams[0] before the next group starts.  The whole
-// run can be captured once into a CUDA graph and replayed with one launch.
+// and joins back into streams[0] before the next group starts.  In the fused
+// launch mode the GEMMs of a wave that share a kernel kind go out as one
+// persistent launch over all their tiles instead.  The whole run can be
+// captured once into a CUDA graph and replayed with one launch.
 //
 // Per GEMM the host encodes two TMA tensor maps (A and B), sizes the
 // persistent grid as min(units, resident CTAs per SM * SMs / rc_div) — the
@@ -50,7 +52,7 @@ struct DeviceState {
   bool init = false;
   int sm_count = 0;
   int* err_word = nullptr;
-  int ctas_per_sm[kNumKinds][2] = {};   // 0 = not yet set up
+  int ctas_per_sm[kNumKinds][2][2] = {};   // [kind][bf16 out][fused]; 0 = not yet set up
 };
 
 std::mutex g_mu;
@@ -61,18 +63,18 @@ goldy_status cuda_fail(cudaError_t e, const char* what) {
   return fail(GOLDY_ERR_CUDA, std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")");
 }
 
-const void* kernel_fn(int kind, int out_bf16) {
+const void* kernel_fn(int kind, int out_bf16, int fused) {
   switch (kind) {
-    case 0: return kernel_fn_k0(out_bf16);
-    case 1: return kernel_fn_k1(out_bf16);
-    case 2: return kernel_fn_k2(out_bf16);
-    case 3: return kernel_fn_k3(out_bf16);
-    case 4: return kernel_fn_k4(out_bf16);
-    case 5: return kernel_fn_k5(out_bf16);
-    case 6: return kernel_fn_k6(out_bf16);
-    case 7: return kernel_fn_k7(out_bf16);
-    case 8: return kernel_fn_k8(out_bf16);
-    case 9: return kernel_fn_k9(out_bf16);
+    case 0: return kernel_fn_k0(out_bf16, fused);
+    case 1: return kernel_fn_k1(out_bf16, fused);
+    case 2: return kernel_fn_k2(out_bf16, fused);
+    case 3: return kernel_fn_k3(out_bf16, fused);
+    case 4: return kernel_fn_k4(out_bf16, fused);
+    case 5: return kernel_fn_k5(out_bf16, fused);
+    case 6: return kernel_fn_k6(out_bf16, fused);
+    case 7: return kernel_fn_k7(out_bf16, fused);
+    case 8: return kernel_fn_k8(out_bf16, fused);
+    case 9: return kernel_fn_k9(out_bf16, fused);
     default: return nullptr;
   }
 }
@@ -104,13 +106,14 @@ goldy_status device_state(DeviceState** out) {
   return GOLDY_OK;
 }
 
-// Resident CTAs per SM of one kernel (kind, dtype) on this device; also opts
-// the kernel into its dynamic shared-memory size the first time.
-goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int* ctas) {
+// Resident CTAs per SM of one kernel (kind, dtype, launch form) on this
+// device; also opts the kernel into its dynamic shared-memory size the first
+// time.
+goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int* ctas) {
   std::lock_guard<std::mutex> lock(g_mu);
-  int& c = d.ctas_per_sm[kind][out_bf16];
+  int& c = d.ctas_per_sm[kind][out_bf16][fused];
   if (c == 0) {
-    const void* fn = kernel_fn(kind, out_bf16);
+    const void* fn = kernel_fn(kind, out_bf16, fused);
     if (!fn) return fail(GOLDY_ERR_UNSUPPORTED, "no kernel for this kind");
     const KindInfo& k = kKinds[kind];
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes(k));
@@ -142,28 +145,18 @@ goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, const void* B, void* C, uint8_t* ws,
-                         cudaStream_t stream) {
+// One GEMM's slot of a launch: tensor maps and work description.
+template <int MAXG>
+goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const void* A, const void* B, void* C,
+                       uint8_t* ws, int32_t unit_begin) {
   const goldy_gemm_desc& g = gp.desc;
-  const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
-  if (g.M == 0 || g.N == 0) return GOLDY_OK;
-  if (g.K == 0) {
-    cudaError_t e = cudaMemset2DAsync(C, size_t(g.ldc) * es, 0, size_t(g.N) * es, size_t(g.M), stream);
-    return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
-  }
   const KindInfo& k = kKinds[gp.kind];
-  const int out_bf16 = g.c_dtype == GOLDY_BF16 ? 1 : 0;
-  int ctas = 0;
-  goldy_status st = kernel_setup(d, gp.kind, out_bf16, &ctas);
+  goldy_status st =
+      encode_2d(&p.tmap_a[j], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(tile_rows(k)));
   if (st != GOLDY_OK) return st;
-
-  LaunchParams<1> p;
-  std::memset(&p, 0, sizeof(p));
-  st = encode_2d(&p.tmap_a[0], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(tile_rows(k)));
+  st = encode_2d(&p.tmap_b[j], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.ldb) * 2, 64, kBlockK);
   if (st != GOLDY_OK) return st;
-  st = encode_2d(&p.tmap_b[0], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.ldb) * 2, 64, kBlockK);
-  if (st != GOLDY_OK) return st;
-  GemmWork& w = p.g[0];
+  GemmWork& w = p.g[j];
   w.c = C;
   w.ldc = g.ldc;
   w.m = int32_t(g.M);
@@ -173,13 +166,40 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   w.tiles_n = int32_t(gp.tiles_n);
   w.split = gp.split;
   w.k_blocks = int32_t(gp.k_blocks);
-  w.unit_begin = 0;
+  w.unit_begin = unit_begin;
   if (gp.split > 1) {
     w.ws_part = reinterpret_cast<float*>(ws + gp.ws_part_off);
     w.ws_cnt = reinterpret_cast<uint32_t*>(ws + gp.ws_cnt_off);
   }
-  p.n_gemms = 1;
+  return GOLDY_OK;
+}
+
+// GEMMs that need no kernel: nothing to write (M or N is 0) or C = 0 (K is 0).
+bool degenerate(const GemmPlan& gp) { return gp.desc.M == 0 || gp.desc.N == 0 || gp.desc.K == 0; }
+
+goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream) {
+  const goldy_gemm_desc& g = gp.desc;
+  if (g.M == 0 || g.N == 0) return GOLDY_OK;
+  const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
+  cudaError_t e = cudaMemset2DAsync(C, size_t(g.ldc) * es, 0, size_t(g.N) * es, size_t(g.M), stream);
+  return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
+}
+
+goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, const void* B, void* C, uint8_t* ws,
+                         cudaStream_t stream) {
+  if (degenerate(gp)) return launch_degenerate(gp, C, stream);
+  const KindInfo& k = kKinds[gp.kind];
+  const int out_bf16 = gp.desc.c_dtype == GOLDY_BF16 ? 1 : 0;
+  int ctas = 0;
+  goldy_status st = kernel_setup(d, gp.kind, out_bf16, 0, &ctas);
+  if (st != GOLDY_OK) return st;
   if (gp.units > int64_t(1) << 30) return fail(GOLDY_ERR_UNSUPPORTED, "too many tiles in one GEMM");
+
+  LaunchParams<1> p;
+  std::memset(&p, 0, sizeof(p));
+  st = fill_slot(p, 0, gp, A, B, C, ws, 0);
+  if (st != GOLDY_OK) return st;
+  p.n_gemms = 1;
   p.total_units = int32_t(gp.units);
   p.err = d.err_word;
 
@@ -187,9 +207,45 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   const int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
   const unsigned grid = unsigned(std::min<int64_t>(gp.units, cap));
   void* args[] = {&p};
-  cudaError_t e = cudaLaunchKernel(kernel_fn(gp.kind, out_bf16), dim3(grid), dim3(kThreads), args,
+  cudaError_t e = cudaLaunchKernel(kernel_fn(gp.kind, out_bf16, 0), dim3(grid), dim3(kThreads), args,
                                    size_t(smem_bytes(k)), stream);
   if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel");
+  return GOLDY_OK;
+}
+
+// One launch over the tiles of `count` (<= kMaxFused) GEMMs of one kind and
+// output dtype.  The grid cap is the sum of the members' own caps (each
+// GO-Kernel keeps the share of the GPU it was tuned for), at most the whole
+// GPU.
+goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* members, int count,
+                          const void* const* A, const void* const* B, void* const* C, uint8_t* ws,
+                          cudaStream_t stream) {
+  const GemmPlan& g0 = s->gemms[members[0]];
+  const KindInfo& k = kKinds[g0.kind];
+  const int out_bf16 = g0.desc.c_dtype == GOLDY_BF16 ? 1 : 0;
+  int ctas = 0;
+  goldy_status st = kernel_setup(d, g0.kind, out_bf16, 1, &ctas);
+  if (st != GOLDY_OK) return st;
+  static thread_local LaunchParams<kMaxFused> p;   // ~5 KB: keep it off the stack
+  std::memset(&p, 0, sizeof(p));
+  int64_t units = 0, cap = 0;
+  for (int j = 0; j < count; ++j) {
+    const GemmPlan& gp = s->gemms[members[j]];
+    st = fill_slot(p, j, gp, A[members[j]], B[members[j]], C[members[j]], ws, int32_t(units));
+    if (st != GOLDY_OK) return st;
+    units += gp.units;
+    cap += std::max<int64_t>(1, int64_t(ctas) * d.sm_count / variant_of(gp.variant).rc_div);
+  }
+  if (units > int64_t(1) << 30) return fail(GOLDY_ERR_UNSUPPORTED, "too many tiles in one launch");
+  p.n_gemms = count;
+  p.total_units = int32_t(units);
+  p.err = d.err_word;
+  cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
+  const unsigned grid = unsigned(std::min<int64_t>(units, cap));
+  void* args[] = {&p};
+  cudaError_t e = cudaLaunchKernel(kernel_fn(g0.kind, out_bf16, 1), dim3(grid), dim3(kThreads), args,
+                                   size_t(smem_bytes(k)), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (fused)");
   return GOLDY_OK;
 }
 
@@ -263,9 +319,55 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
 
+  auto hook = [&](void* const* evs, const int* members, int n, cudaStream_t stream) -> goldy_status {
+    if (!evs) return GOLDY_OK;
+    for (int j = 0; j < n; ++j) {
+      cudaError_t e = record_hook(evs[members[j]], stream);
+      if (e != cudaSuccess) return cuda_fail(e, "timing event");
+    }
+    return GOLDY_OK;
+  };
+  const bool fused = (s->flags & GOLDY_PLAN_FUSED) != 0;
+
   for (const Group& grp : s->groups) {
+    // Launch sets.  Streams mode: one per GEMM, on the GEMM's slot.  Fused
+    // mode: the group's members taken CD at a time form waves; in a wave, the
+    // GEMMs of one kind and output dtype share a launch on the slot of the
+    // first of them.
+    struct LaunchSet {
+      int slot, n, degenerate;
+      int members[kMaxFused];
+    };
+    LaunchSet sets[GOLDY_MAX_GEMMS];
+    int n_sets = 0;
+    const int size = int(grp.members.size());
+    const int wave = fused ? std::max(1, grp.cd) : 1;
+    for (int w0 = 0; w0 < size; w0 += wave) {
+      const int first_set = n_sets;
+      for (int j = w0; j < std::min(size, w0 + wave); ++j) {
+        const int i = grp.members[j];
+        const GemmPlan& gp = s->gemms[i];
+        int target = -1;
+        if (fused && !degenerate(gp))
+          for (int t = first_set; t < n_sets; ++t) {
+            const GemmPlan& g0 = s->gemms[sets[t].members[0]];
+            if (!sets[t].degenerate && sets[t].n < kMaxFused && g0.kind == gp.kind &&
+                g0.desc.c_dtype == gp.desc.c_dtype) {
+              target = t;
+              break;
+            }
+          }
+        if (target < 0) {
+          target = n_sets++;
+          sets[target].slot = gp.slot;
+          sets[target].n = 0;
+          sets[target].degenerate = degenerate(gp) ? 1 : 0;
+        }
+        sets[target].members[sets[target].n++] = i;
+      }
+    }
     uint32_t used = 0;
-    for (int i : grp.members) used |= 1u << s->gemms[i].slot;
+    for (int t = 0; t < n_sets; ++t) used |= 1u << sets[t].slot;
     const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
     if (side) {
       cudaError_t e = cudaEventRecord(rt->fork, main);
@@ -276,19 +378,20 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
           if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
         }
     }
-    for (int i : grp.members) {
-      const GemmPlan& gp = s->gemms[i];
-      cudaStream_t st_i = static_cast<cudaStream_t>(streams[gp.slot]);
-      if (opts && opts->ev_begin) {
-        cudaError_t e = record_hook(opts->ev_begin[i], st_i);
-        if (e != cudaSuccess) return cuda_fail(e, "timing event");
-      }
-      st = launch_gemm(*d, gp, A[i], B[i], C[i], ws, st_i);
+    for (int t = 0; t < n_sets; ++t) {
+      const LaunchSet& ls = sets[t];
+      cudaStream_t stream = static_cast<cudaStream_t>(streams[ls.slot]);
+      st = hook(opts ? opts->ev_begin : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
-      if (opts && opts->ev_end) {
-        cudaError_t e = record_hook(opts->ev_end[i], st_i);
-        if (e != cudaSuccess) return cuda_fail(e, "timing event");
+      if (ls.n == 1) {
+        const int i = ls.members[0];
+        st = launch_gemm(*d, s->gemms[i], A[i], B[i], C[i], ws, stream);
+      } else {
+        st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream);
       }
+      if (st != GOLDY_OK) return st;
+      st = hook(opts ? opts->ev_end : nullptr, ls.members, ls.n, stream);
+      if (st != GOLDY_OK) return st;
     }
     if (side) {
       for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
@@ -380,7 +483,7 @@ extern "C" goldy_status goldy_device_info(int variant_id, int* sm_count, int* ct
   if (st != GOLDY_OK) return st;
   const Variant v = variant_of(variant_id);
   int ctas = 0;
-  st = kernel_setup(*d, v.kind, 0, &ctas);
+  st = kernel_setup(*d, v.kind, 0, 0, &ctas);
   if (st != GOLDY_OK) return st;
   if (sm_count) *sm_count = d->sm_count;
   if (ctas_per_sm) *ctas_per_sm = ctas;

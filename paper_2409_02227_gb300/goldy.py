@@ -33,6 +33,7 @@ GOLDY_PLAN_SEQUENTIAL = 1
 GOLDY_PLAN_DEFAULT = 2
 GOLDY_PLAN_GO = 3
 GOLDY_PLAN_FORCE_CD = 4
+GOLDY_PLAN_FUSED = 0x10
 GOLDY_MAX_GEMMS = 64
 GOLDY_MAX_STREAMS = 16
 
@@ -90,7 +91,7 @@ def _load():
         "goldy_lut_free": ([P], None),
         "goldy_bucket_key": ([DP, ctypes.POINTER(U32)], I),
         "goldy_plan": ([DP, I, P, I, PP], I),
-        "goldy_schedule_build": ([DP, I, IP, IP, IP, PP], I),
+        "goldy_schedule_build": ([DP, I, IP, IP, IP, I, PP], I),
         "goldy_schedule_query": ([P, IP, IP, IP, ctypes.POINTER(SZ)], I),
         "goldy_schedule_entry": ([P, I, IP, IP, IP, IP], I),
         "goldy_schedule_serialize": ([P, P, SZ, ctypes.POINTER(SZ)], I),
@@ -216,12 +217,12 @@ def goldy_plan(descs: Sequence[goldy_gemm_desc], lut: Lut, flags: int = GOLDY_PL
 
 
 def goldy_schedule_build(descs: Sequence[goldy_gemm_desc], group_of: Sequence[int],
-                         variant_of: Sequence[int], slot_of: Sequence[int]) -> Schedule:
+                         variant_of: Sequence[int], slot_of: Sequence[int], flags: int = 0) -> Schedule:
     n = len(descs)
     IA = ctypes.c_int * max(1, n)
     out = ctypes.c_void_p()
     _check(_lib.goldy_schedule_build(_descs(descs), n, IA(*group_of), IA(*variant_of), IA(*slot_of),
-                                     ctypes.byref(out)), "goldy_schedule_build")
+                                     int(flags), ctypes.byref(out)), "goldy_schedule_build")
     return Schedule(out)
 
 

@@ -136,6 +136,10 @@ def test_schedule_build_and_query():
         G.goldy_schedule_build(descs, [0, 0, 0], [0, 0, 0], [0, 0, 16])
     with pytest.raises(G.GoldyError):
         G.goldy_schedule_entry(s, 3)
+    with pytest.raises(G.GoldyError):
+        G.goldy_schedule_build(descs, [0, 0, 1], [0, 9, 80], [0, 3, 0], flags=1)
+    f = G.goldy_schedule_build(descs, [0, 0, 1], [0, 9, 80], [0, 3, 0], flags=G.GOLDY_PLAN_FUSED)
+    assert G.goldy_schedule_serialize(f)[20:24] == bytes([0x10, 0, 0, 0])
 
 
 def test_bucket_key_matches_reference():

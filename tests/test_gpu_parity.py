@@ -178,3 +178,78 @@ def test_config_hetero_pair_sampled(cuda_ok):
 
 def test_device_error_word_clear(cuda_ok):
     assert G.goldy_device_error(clear=False) == 0
+
+
+def _run_sched(As, Bs, outs, variants, groups, slots, flags):
+    descs = [G.desc(a.shape[0], b.shape[1], a.shape[1], o) for a, b, o in zip(As, Bs, outs)]
+    s = G.goldy_schedule_build(descs, groups, variants, slots, flags)
+    L = Launch(s, As, Bs, outs)
+    L.run()
+    return L.results()
+
+
+def _same_bytes(x, y):
+    if x.dtype == torch.bfloat16:
+        return torch.equal(x.view(torch.int16), y.view(torch.int16))
+    return torch.equal(x, y)
+
+
+def test_fused_launch_matches_streams(cuda_ok):
+    # four same-kind GEMMs of different shapes and splits in one launch
+    shapes = [(128, 1024, 4096), (100, 512, 1024), (256, 320, 2048), (128, 1024, 4096)]
+    A, B = zip(*[inputs(M, N, K, seed=700 + i, dist="normal", scale=0.05) for i, (M, N, K) in enumerate(shapes)])
+    vs = [vid(1, 4, 4), vid(1, 2, 2), vid(1, 1, 1), vid(1, 8, 4)]
+    outs = [BF16] * 4
+    ref = _run_sched(list(A), list(B), outs, vs, [0] * 4, [0, 1, 2, 3], 0)
+    got = _run_sched(list(A), list(B), outs, vs, [0] * 4, [0, 1, 2, 3], G.GOLDY_PLAN_FUSED)
+    for i in range(4):
+        check_close(got[i], A[i], B[i], f"fused gemm {i}")
+        assert _same_bytes(got[i], ref[i])
+
+
+def test_fused_mixed_kinds_waves_and_degenerate(cuda_ok):
+    # group 0: CD 3 over 5 members -> waves {0,1,2} (three kinds, three launches) and
+    # {3,4} (one kind: one fused launch); group 1: a K = 0 member next to a real one
+    shapes = [(64, 4096, 512), (200, 320, 448), (40, 296, 320), (200, 320, 448), (130, 256, 1024),
+              (70, 136, 0), (33, 64, 64)]
+    outs = [F32, F32, BF16, F32, F32, F32, F32]
+    A, B = [], []
+    for i, (M, N, K) in enumerate(shapes):
+        if K == 0:
+            A.append(torch.zeros((M, 0), dtype=torch.bfloat16))
+            B.append(torch.zeros((0, N), dtype=torch.bfloat16))
+        else:
+            a, b = inputs(M, N, K, seed=800 + i)
+            A.append(a)
+            B.append(b)
+    vs = [vid(7, 2, 4), vid(3, 1, 2), vid(6, 1, 4), vid(3, 2, 2), vid(3, 4, 4), vid(2), vid(2)]
+    groups = [0, 0, 0, 0, 0, 1, 1]
+    slots = [0, 1, 2, 0, 1, 0, 1]
+    descs = [G.desc(a.shape[0], b.shape[1], a.shape[1], o, lda=max(8, a.shape[1])) for a, b, o in zip(A, B, outs)]
+    res = {}
+    for flags in (0, G.GOLDY_PLAN_FUSED):
+        s = G.goldy_schedule_build(descs, groups, vs, slots, flags)
+        L = Launch(s, A, B, outs)
+        L.run()
+        res[flags] = L.results()
+    for i in range(7):
+        if shapes[i][2] == 0:
+            assert torch.equal(res[G.GOLDY_PLAN_FUSED][i], torch.zeros_like(res[0][i]))
+            continue
+        check_close(res[G.GOLDY_PLAN_FUSED][i], A[i], B[i], f"fused mixed {i}")
+        assert _same_bytes(res[G.GOLDY_PLAN_FUSED][i], res[0][i])
+
+
+def test_fused_plan_graph_replay(cuda_ok):
+    st = wl.make_config("lstm_gates")
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    v = vid(7, 2, 4)
+    s = G.goldy_schedule_build(descs, [0] * 8, [v] * 8, list(range(8)), G.GOLDY_PLAN_FUSED)
+    L = Launch(s, st.a, st.b, [s_.out_dtype for s_ in st.specs])
+    g = L.graph()
+    for _ in range(3):
+        G.goldy_graph_launch(g, L.streams[0].cuda_stream)
+    torch.cuda.current_stream().wait_stream(L.streams[0])
+    got = L.results()
+    for i in range(8):
+        check_close(got[i], st.a[i], st.b[i], f"lstm fused {i}")

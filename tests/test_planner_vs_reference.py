@@ -32,7 +32,9 @@ def random_desc(rng, shapes):
 def flags_for(rng):
     pol = rng.choice([0, 0, 0, 0, 1, 2, 3, 4])
     if pol == 4:
-        return pol | (rng.randint(1, 20) << 8)
+        pol |= rng.randint(1, 20) << 8
+    if rng.random() < 0.3:
+        pol |= G.GOLDY_PLAN_FUSED
     return pol
 
 
