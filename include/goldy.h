@@ -212,6 +212,17 @@ goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void
 typedef struct goldy_run_opts {
   void* const* ev_begin;
   void* const* ev_end;
+  /* Optional device buffer of unsigned 64-bit words for a phase trace: every
+   * CTA of every GO-Kernel launch writes 16 words at trace[cta * 16 + k]
+   * (k: 0 entry, 1 set-up done, 2 first TMA load, 3 first full stage seen by
+   * the MMA thread, 4 first accumulator committed, 5 first accumulator seen
+   * by the epilogue, 6 split-K partial stored, 7 split-K arrival counted,
+   * 8 first unit stored, 9 exit — %globaltimer nanoseconds; 14 units this CTA
+   * processed; 15 SM id).  Size it for the largest grid (trace_ctas CTAs);
+   * launches of one run share it, so use it on single-launch schedules.
+   * Null: no tracing. */
+  void* trace;
+  size_t trace_ctas;
 } goldy_run_opts;
 
 /* goldy_run with options; opts may be null (then identical to goldy_run). */

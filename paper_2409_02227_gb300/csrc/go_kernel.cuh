@@ -63,6 +63,24 @@ struct LaunchParams {
   int32_t n_gemms;
   int32_t total_units;
   int* err;                   // device error word (first failure wins)
+  unsigned long long* trace;  // optional phase trace, kTracePerCta stamps per CTA (null: off)
+};
+
+// Phase trace (optional, for profiling): %globaltimer stamps per CTA.
+enum : int {
+  kTrStart = 0,        // kernel entry
+  kTrSetup = 1,        // barriers initialised, tensor memory allocated
+  kTrFirstLoad = 2,    // producer issued its first TMA load
+  kTrFirstFull = 3,    // MMA thread saw its first full stage
+  kTrFirstMmaDone = 4, // MMA thread committed its first accumulator
+  kTrFirstAcc = 5,     // epilogue saw its first accumulator
+  kTrPartials = 6,     // split-K: partial tile stored and fenced
+  kTrArrived = 7,      // split-K: arrival counter bumped
+  kTrFirstStore = 8,   // epilogue finished its first unit
+  kTrEnd = 9,          // all roles done
+  kTrUnits = 14,       // units processed by this CTA
+  kTrSm = 15,          // SM id
+  kTracePerCta = 16,
 };
 
 enum : int {
@@ -91,6 +109,10 @@ __device__ __forceinline__ UnitCoord decode_unit(const LaunchParams<MAXG>& p, in
   c.kb0 = (c.s * w.k_blocks) / w.split;
   c.kb1 = ((c.s + 1) * w.k_blocks) / w.split;
   return c;
+}
+
+__device__ __forceinline__ void trace_stamp(unsigned long long* trace, int slot) {
+  if (trace) trace[blockIdx.x * kTracePerCta + slot] = ptx::global_timer();
 }
 
 __device__ __forceinline__ void raise_error(int* err, volatile int* abort_flag, int code) {
@@ -196,8 +218,15 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
   const uint32_t tiles_base = ptx::smem_u32(smem);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  unsigned long long* const trace = p.trace;
 
   if (threadIdx.x == 0) {
+    trace_stamp(trace, kTrStart);
+    if (trace) {
+      uint32_t sm;
+      asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+      trace[blockIdx.x * kTracePerCta + kTrSm] = sm;
+    }
     for (int s = 0; s < STAGES; ++s) {
       ptx::mbar_init(ptx::smem_u32(&full[s]), 1);
       ptx::mbar_init(ptx::smem_u32(&empty[s]), 1);
@@ -220,6 +249,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -256,6 +286,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
             for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_2d(xs + j * 8192, tb, fb, n0 + 64 * j, k0);
             ptx::tma_load_2d(ys, ta, fb, k0, m0);
           }
+          if (issued == 0) trace_stamp(trace, kTrFirstLoad);
           issued |= 1u << stage;
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -291,6 +322,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
             break;
           }
           ptx::tc_fence_after();
+          if (!any) trace_stamp(trace, kTrFirstFull);
           const uint32_t xs = tiles_base + stage * STAGE_BYTES;
           const uint32_t ys = xs + X_BYTES;
 #pragma unroll
@@ -314,6 +346,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
         }
         if (!ok) break;
         ptx::mma_commit(ptx::smem_u32(&tfull[acc]));        // accumulator complete
+        if (u == int(blockIdx.x)) trace_stamp(trace, kTrFirstMmaDone);
         if (++acc == ACC) {
           acc = 0;
           acc_phase ^= 1;
@@ -343,6 +376,8 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
         break;
       }
       ptx::tc_fence_after();
+      const bool first_unit = (u == int(blockIdx.x));
+      if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
       const GemmWork& w = p.g[c.g];
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
@@ -379,8 +414,10 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
         __threadfence();
         ptx::named_bar_sync(1, 128);
         if (et == 0) {
+          if (first_unit) trace_stamp(trace, kTrPartials);
           const uint32_t old = atomicAdd(&w.ws_cnt[c.tile], 1u);
           *last_flag = (old == uint32_t(w.split - 1)) ? 1 : 0;
+          if (first_unit) trace_stamp(trace, kTrArrived);
         }
         ptx::named_bar_sync(1, 128);
         if (*last_flag) {
@@ -416,6 +453,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
           if (et == 0) w.ws_cnt[c.tile] = 0u;     // leave the counter zeroed for the next run
         }
       }
+      if (first_unit && et == 0) trace_stamp(trace, kTrFirstStore);
       ptx::tc_fence_before();
       ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));
       if (++acc == ACC) {
@@ -426,6 +464,14 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
   }
 
   __syncthreads();
+  if (threadIdx.x == 0) {
+    trace_stamp(trace, kTrEnd);
+    if (trace) {
+      int n = 0;
+      for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) ++n;
+      trace[blockIdx.x * kTracePerCta + kTrUnits] = n;
+    }
+  }
   if (warp == 1) {
     __syncwarp();
     ptx::tc_fence_after();

@@ -185,6 +185,14 @@ goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream)
   return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
 }
 
+// Phase-trace buffer of the current goldy_run_ex call (null: off).
+thread_local unsigned long long* t_trace = nullptr;
+thread_local size_t t_trace_ctas = 0;
+
+unsigned long long* trace_for(unsigned grid) {
+  return (t_trace && grid <= t_trace_ctas) ? t_trace : nullptr;
+}
+
 goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, const void* B, void* C, uint8_t* ws,
                          cudaStream_t stream) {
   if (degenerate(gp)) return launch_degenerate(gp, C, stream);
@@ -206,6 +214,7 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   const Variant v = variant_of(gp.variant);
   const int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
   const unsigned grid = unsigned(std::min<int64_t>(gp.units, cap));
+  p.trace = trace_for(grid);
   void* args[] = {&p};
   cudaError_t e = cudaLaunchKernel(kernel_fn(gp.kind, out_bf16, 0), dim3(grid), dim3(kThreads), args,
                                    size_t(smem_bytes(k)), stream);
@@ -242,6 +251,7 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.err = d.err_word;
   cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
   const unsigned grid = unsigned(std::min<int64_t>(units, cap));
+  p.trace = trace_for(grid);
   void* args[] = {&p};
   cudaError_t e = cudaLaunchKernel(kernel_fn(g0.kind, out_bf16, 1), dim3(grid), dim3(kThreads), args,
                                    size_t(smem_bytes(k)), stream);
@@ -319,6 +329,8 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
 
+  t_trace = opts ? static_cast<unsigned long long*>(opts->trace) : nullptr;
+  t_trace_ctas = opts ? opts->trace_ctas : 0;
   auto hook = [&](void* const* evs, const int* members, int n, cudaStream_t stream) -> goldy_status {
     if (!evs) return GOLDY_OK;
     for (int j = 0; j < n; ++j) {
@@ -402,6 +414,8 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
         }
     }
   }
+  t_trace = nullptr;
+  t_trace_ctas = 0;
   return ok();
 }
 

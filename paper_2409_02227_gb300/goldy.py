@@ -58,7 +58,8 @@ class goldy_gemm_desc(ctypes.Structure):
 
 
 class goldy_run_opts(ctypes.Structure):
-    _fields_ = [("ev_begin", ctypes.POINTER(ctypes.c_void_p)), ("ev_end", ctypes.POINTER(ctypes.c_void_p))]
+    _fields_ = [("ev_begin", ctypes.POINTER(ctypes.c_void_p)), ("ev_end", ctypes.POINTER(ctypes.c_void_p)),
+                ("trace", ctypes.c_void_p), ("trace_ctas", ctypes.c_size_t)]
 
 
 class goldy_variant_info(ctypes.Structure):
@@ -266,8 +267,11 @@ def goldy_graph_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Seque
     return Graph(out)
 
 
-def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]]):
+def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]], trace: int = 0,
+          trace_ctas: int = 0):
     o = goldy_run_opts()
+    o.trace = int(trace) or None
+    o.trace_ctas = int(trace_ctas)
     keep = []
     if ev_begin is not None:
         arr = _ptrs(ev_begin)
@@ -282,9 +286,10 @@ def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]]):
 
 def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
                  workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
-                 ev_end: Optional[Sequence[int]] = None) -> None:
-    """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints)."""
-    o, _keep = _opts(ev_begin, ev_end)
+                 ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0) -> None:
+    """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints)
+    and an optional device phase-trace buffer (see goldy_run_opts)."""
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas)
     _check(_lib.goldy_run_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                              int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o)),
            "goldy_run_ex")

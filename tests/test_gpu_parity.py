@@ -253,3 +253,28 @@ def test_fused_plan_graph_replay(cuda_ok):
     got = L.results()
     for i in range(8):
         check_close(got[i], st.a[i], st.b[i], f"lstm fused {i}")
+
+
+def test_phase_trace_is_consistent(cuda_ok):
+    # the optional per-CTA trace: every CTA stamps its phases in order and the
+    # units it reports add up to the launch's units
+    shapes = [(128, 1024, 4096)] * 2
+    A, B = zip(*[inputs(M, N, K, seed=900 + i, dist="normal", scale=0.05) for i, (M, N, K) in enumerate(shapes)])
+    v = vid(1, 4, 1)
+    descs = [G.desc(M, N, K, BF16) for (M, N, K) in shapes]
+    s = G.goldy_schedule_build(descs, [0, 0], [v, v], [0, 1], G.GOLDY_PLAN_FUSED)
+    L = Launch(s, list(A), list(B), [BF16, BF16])
+    trace = torch.zeros(512 * 16, dtype=torch.int64, device="cuda")
+    A_, B_, C_ = L.ptrs()
+    G.goldy_run_ex(s, A_, B_, C_, L.ws.data_ptr(), L.ws_bytes, [x.cuda_stream for x in L.streams],
+                   trace=trace.data_ptr(), trace_ctas=512)
+    got = L.results()
+    for i in range(2):
+        check_close(got[i], A[i], B[i], f"traced {i}")
+    t = trace.view(512, 16).cpu()
+    rows = t[t[:, 0] != 0]
+    assert rows.shape[0] > 0
+    assert int(rows[:, 14].sum()) == 2 * 16 * 4                  # 16 tiles x split 4 per GEMM
+    for r in rows.tolist():
+        assert r[0] <= r[1] <= r[2] and r[1] <= r[3] <= r[4] and r[5] <= r[8] <= r[9]
+        assert r[6] <= r[7] and r[4] <= r[5]
