@@ -184,8 +184,8 @@ struct TmemCols {
   static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
 };
 
-template <int MMA_N, bool SWAP, int STAGES, int ACC, bool OUT_BF16, int MAXG>
-__global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__ LaunchParams<MAXG> p) {
+template <int MMA_N, bool SWAP, int STAGES, int ACC, bool OUT_BF16, int MAXG, int MIN_CTAS>
+__global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_constant__ LaunchParams<MAXG> p) {
   constexpr int X_BYTES = 128 * 64 * 2;              // MMA operand A: 128 rows x 64 K
   constexpr int Y_BYTES = MMA_N * 64 * 2;            // MMA operand B: MMA_N rows x 64 K
   constexpr int STAGE_BYTES = X_BYTES + Y_BYTES;
@@ -222,6 +222,12 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
 
   if (threadIdx.x == 0) {
     trace_stamp(trace, kTrStart);
+    // start fetching the TMA descriptors before anything else: the first
+    // load waits on them
+    for (int g = 0; g < p.n_gemms; ++g) {
+      ptx::prefetch_tensormap(&p.tmap_a[g]);
+      ptx::prefetch_tensormap(&p.tmap_b[g]);
+    }
     if (trace) {
       uint32_t sm;
       asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
@@ -254,10 +260,6 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ producer
-      for (int g = 0; g < p.n_gemms; ++g) {
-        ptx::prefetch_tensormap(&p.tmap_a[g]);
-        ptx::prefetch_tensormap(&p.tmap_b[g]);
-      }
       int stage = 0;
       uint32_t phase = 0, issued = 0, last_phase = 0;
       bool ok = true;
@@ -431,20 +433,36 @@ __global__ void __launch_bounds__(192, 1) go_gemm_kernel(const __grid_constant__
             float v[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+            // two splits' partials are loaded before either is added, so their
+            // loads are in flight together; the sum runs in split order
+            // 0, 1, ..., S-1 (the own split's values come from tensor memory)
 #pragma unroll 1
-            for (int s2 = 0; s2 < w.split; ++s2) {
-              if (s2 == c.s) {
+            for (int s2 = 0; s2 < w.split; s2 += 2) {
+              const bool has_b = s2 + 1 < w.split;
+              float4 ta[8], tb[8];
+              const float4* pa = part_base + size_t(c.tile * w.split + s2) * TILE_F4;
+              const float4* pb = part_base + size_t(c.tile * w.split + s2 + 1) * TILE_F4;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(raw[j]);
-              } else {
-                const float4* other = part_base + size_t(c.tile * w.split + s2) * TILE_F4;
+              for (int j4 = 0; j4 < 8; ++j4) {
+                const float4 own = make_float4(__uint_as_float(raw[4 * j4]), __uint_as_float(raw[4 * j4 + 1]),
+                                               __uint_as_float(raw[4 * j4 + 2]), __uint_as_float(raw[4 * j4 + 3]));
+                ta[j4] = (s2 == c.s) ? own : __ldcg(&pa[((c0 / 4) + j4) * 128 + r]);
+                tb[j4] = (!has_b || s2 + 1 == c.s) ? own : __ldcg(&pb[((c0 / 4) + j4) * 128 + r]);
+              }
+#pragma unroll
+              for (int j4 = 0; j4 < 8; ++j4) {
+                v[4 * j4] += ta[j4].x;
+                v[4 * j4 + 1] += ta[j4].y;
+                v[4 * j4 + 2] += ta[j4].z;
+                v[4 * j4 + 3] += ta[j4].w;
+              }
+              if (has_b) {
 #pragma unroll
                 for (int j4 = 0; j4 < 8; ++j4) {
-                  const float4 t = __ldcg(&other[((c0 / 4) + j4) * 128 + r]);
-                  v[4 * j4] += t.x;
-                  v[4 * j4 + 1] += t.y;
-                  v[4 * j4 + 2] += t.z;
-                  v[4 * j4 + 3] += t.w;
+                  v[4 * j4] += tb[j4].x;
+                  v[4 * j4 + 1] += tb[j4].y;
+                  v[4 * j4 + 2] += tb[j4].z;
+                  v[4 * j4 + 3] += tb[j4].w;
                 }
               }
             }

@@ -23,13 +23,13 @@ const void* GOLDY_CAT(kernel_fn_k, GOLDY_KIND)(int out_bf16, int fused) {
   if (fused) {
     if (out_bf16)
       return reinterpret_cast<const void*>(
-          &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, kMaxFused>);
+          &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, kMaxFused, kK.ctas_per_sm>);
     return reinterpret_cast<const void*>(
-        &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, kMaxFused>);
+        &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, kMaxFused, kK.ctas_per_sm>);
   }
   if (out_bf16)
-    return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, 1>);
-  return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, 1>);
+    return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, 1, kK.ctas_per_sm>);
+  return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, 1, kK.ctas_per_sm>);
 }
 
 }  // namespace goldy

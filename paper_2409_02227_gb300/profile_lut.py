@@ -11,9 +11,10 @@ list:
          contention for it is only seen in step 2) — and keep the fastest per
          constraint;
   step 2 (concurrent benchmarking): for each concurrency degree CD in
-         {2, 4, 8, 16}, co-run CD copies of the GEMM (distinct buffers, one
-         stream each) with each step-1 winner; the fastest is the GO-Kernel
-         for that CD.  The CD-1 kernel is the whole-GPU winner (the
+         {2, 4, 8, 16}, co-run CD copies of the GEMM (distinct buffers) with
+         each step-1 winner, launched the way the library will launch them
+         (one fused launch by default, or one stream each); the fastest is
+         the GO-Kernel for that CD.  The CD-1 kernel is the whole-GPU winner (the
          isolation-tuned kernel);
   preferred CD: speedup(CD) = CD * T(1) / T(CD) over running the copies one
          after another; the largest wins, but sequential (CD 1) unless some
@@ -119,10 +120,12 @@ class Bench:
             self.ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device="cuda")
         return self.ws
 
-    def time_us(self, variant: int, copies: int, concurrent: bool, target_us: float = 2000.0) -> float:
+    def time_us(self, variant: int, copies: int, concurrent: bool, target_us: float = 2000.0,
+                fused: bool = True) -> float:
         d = G.desc(self.M, self.N, self.K, self.out)
         slots = list(range(copies)) if concurrent else [0] * copies
-        sched = G.goldy_schedule_build([d] * copies, [0] * copies, [variant] * copies, slots)
+        sched = G.goldy_schedule_build([d] * copies, [0] * copies, [variant] * copies, slots,
+                                       G.GOLDY_PLAN_FUSED if fused else 0)
         _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
         ws = self._workspace(ws_bytes)
         torch.cuda.synchronize()
@@ -154,7 +157,7 @@ class Bench:
         return samples[len(samples) // 2]
 
 
-def profile_bucket(key, sm_count: int, log) -> dict:
+def profile_bucket(key, sm_count: int, log, fused: bool = True) -> dict:
     M, N, K, out = bucket_shape(key)
     bench = Bench(M, N, K, out)
     cands = candidates(M, N, K, sm_count)
@@ -164,7 +167,7 @@ def profile_bucket(key, sm_count: int, log) -> dict:
         best = None
         for kind, split in cands:
             v = G.variant_id(kind, split, rc)
-            t = bench.time_us(v, 1, True)
+            t = bench.time_us(v, 1, True, fused=fused)
             rows.append({"step": 1, "rc": rc, "variant": v, "us": t})
             if best is None or t < best[0]:
                 best = (t, v)
@@ -175,7 +178,7 @@ def profile_bucket(key, sm_count: int, log) -> dict:
         best = None
         for rc in RC_DIVS:
             v = winners[rc][1]
-            t = bench.time_us(v, cd, True)
+            t = bench.time_us(v, cd, True, fused=fused)
             rows.append({"step": 2, "cd": cd, "rc": rc, "variant": v, "us": t})
             if best is None or t < best[0]:
                 best = (t, v)
@@ -183,7 +186,7 @@ def profile_bucket(key, sm_count: int, log) -> dict:
         t_cd[cd] = best[0]
     speedup = {cd: cd * t_cd[1] / t_cd[cd] for cd in CD_CLASSES}
     pref = preferred_cd(speedup)
-    rec = {"key": list(key), "shape": [M, N, K, out], "pref_cd": pref,
+    rec = {"key": list(key), "shape": [M, N, K, out], "pref_cd": pref, "launch": "fused" if fused else "streams",
            "variants": [go[c] for c in CD_CLASSES], "t_us": {str(c): t_cd[c] for c in CD_CLASSES},
            "speedup": {str(c): speedup[c] for c in CD_CLASSES}, "rows": rows}
     log.write(json.dumps(rec) + "\n")
@@ -221,6 +224,8 @@ def main(argv=None) -> int:
     ap.add_argument("--sweep", action="store_true", help="buckets of the 64 randomized sets")
     ap.add_argument("--keys", nargs="*", default=[], help="extra buckets lm,ln,lk,out")
     ap.add_argument("--time-budget", type=float, default=1e9, help="stop starting buckets after this many seconds")
+    ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
+                    help="launch mode the co-runs of step 2 use (the mode the table will be used with)")
     args = ap.parse_args(argv)
     os.makedirs(args.out, exist_ok=True)
     keys = []
@@ -246,7 +251,7 @@ def main(argv=None) -> int:
                 print(f"time budget reached after {i} buckets", flush=True)
                 break
             tb = time.time()
-            rec = profile_bucket(key, sm_count, log)
+            rec = profile_bucket(key, sm_count, log, fused=args.launch == "fused")
             done[key] = rec
             print(f"[{i + 1}/{len(keys)}] {key} shape {rec['shape']} pref {rec['pref_cd']} "
                   f"variants {rec['variants']} ({time.time() - tb:.1f}s)", flush=True)
