@@ -64,6 +64,8 @@ struct LaunchParams {
   int32_t total_units;
   int* err;                   // device error word (first failure wins)
   unsigned long long* trace;  // optional phase trace, kTracePerCta stamps per CTA (null: off)
+  int32_t cluster;            // 0, or the split-K factor S of every GEMM in the launch when the
+                              // launch is made of clusters of S CTAs (the splits of one tile)
 };
 
 // Phase trace (optional, for profiling): %globaltimer stamps per CTA.
@@ -87,6 +89,7 @@ enum : int {
   kErrProducerWait = 1,
   kErrMmaWait = 2,
   kErrEpilogueWait = 3,
+  kErrClusterWait = 4,
 };
 
 struct UnitCoord {
@@ -178,6 +181,95 @@ __device__ __forceinline__ void store_chunk(const GemmWork& w, int m0, int n0, i
   }
 }
 
+// Store 4 consecutive accumulator columns (acc_col .. acc_col+3) of
+// accumulator row acc_row, mapped to C as in store_chunk.
+template <bool SWAP, bool OUT_BF16>
+__device__ __forceinline__ void store_quad(const GemmWork& w, int m0, int n0, int acc_row, int acc_col, float4 a) {
+  const float v[4] = {a.x, a.y, a.z, a.w};
+  if (!SWAP) {
+    const int64_t row = int64_t(m0) + acc_row;
+    if (row >= w.m) return;
+    const int col0 = n0 + acc_col;
+    if (OUT_BF16) {
+      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(w.c) + row * w.ldc + col0;
+      if (col0 + 4 <= w.n && (reinterpret_cast<uintptr_t>(dst) & 7) == 0) {
+        __nv_bfloat162 h0 = __floats2bfloat162_rn(v[0], v[1]);
+        __nv_bfloat162 h1 = __floats2bfloat162_rn(v[2], v[3]);
+        uint2 pk;
+        pk.x = *reinterpret_cast<uint32_t*>(&h0);
+        pk.y = *reinterpret_cast<uint32_t*>(&h1);
+        *reinterpret_cast<uint2*>(dst) = pk;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (col0 + j < w.n) dst[j] = __float2bfloat16_rn(v[j]);
+      }
+    } else {
+      float* dst = static_cast<float*>(w.c) + row * w.ldc + col0;
+      if (col0 + 4 <= w.n && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+        *reinterpret_cast<float4*>(dst) = a;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (col0 + j < w.n) dst[j] = v[j];
+      }
+    }
+  } else {
+    const int64_t col = int64_t(n0) + acc_row;
+    if (col >= w.n) return;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int64_t row = int64_t(m0) + acc_col + j;
+      if (row < w.m) {
+        if (OUT_BF16)
+          static_cast<__nv_bfloat16*>(w.c)[row * w.ldc + col] = __float2bfloat16_rn(v[j]);
+        else
+          static_cast<float*>(w.c)[row * w.ldc + col] = v[j];
+      }
+    }
+  }
+}
+
+// Cluster split-K: this CTA (split `rank` of S) sums rows rank*128/S ..
+// (rank+1)*128/S - 1 of the tile over all S partial tiles, in split order
+// 0, 1, ..., S-1, and stores them.  Partial layout: [chunk][float4][row].
+// Per batch, IB items x S partials are loaded before any is added.
+template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
+__device__ __forceinline__ void reduce_slice(const GemmWork& w, const float4* tile_parts, int rank, int m0, int n0,
+                                             int t) {
+  constexpr int R = 128 / S;
+  constexpr int COLS4 = MMA_N / 4;
+  constexpr int PER_THREAD = R * COLS4 / 128;
+  constexpr int IB = (16 / S < PER_THREAD) ? 16 / S : PER_THREAD;
+  constexpr int TILE_F4 = 128 * MMA_N / 4;
+  static_assert(PER_THREAD >= 1 && PER_THREAD % IB == 0, "reduce tiling");
+  const int r0 = rank * R;
+#pragma unroll 1
+  for (int k0 = 0; k0 < PER_THREAD; k0 += IB) {
+    float4 vals[IB][S];
+#pragma unroll
+    for (int b = 0; b < IB; ++b) {
+      const int i = t + 128 * (k0 + b);
+      const int off = (i / R) * 128 + r0 + (i % R);
+#pragma unroll
+      for (int s2 = 0; s2 < S; ++s2) vals[b][s2] = __ldcg(&tile_parts[size_t(s2) * TILE_F4 + off]);
+    }
+#pragma unroll
+    for (int b = 0; b < IB; ++b) {
+      const int i = t + 128 * (k0 + b);
+      float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+      for (int s2 = 0; s2 < S; ++s2) {
+        a.x += vals[b][s2].x;
+        a.y += vals[b][s2].y;
+        a.z += vals[b][s2].z;
+        a.w += vals[b][s2].w;
+      }
+      store_quad<SWAP, OUT_BF16>(w, m0, n0, r0 + (i % R), 4 * (i / R), a);
+    }
+  }
+}
+
 template <int MMA_N, int ACC>
 struct TmemCols {
   static constexpr uint32_t need = uint32_t(MMA_N * ACC);
@@ -211,7 +303,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   uint64_t* tfull = bars + 2 * STAGES;
   uint64_t* tempty = bars + 2 * STAGES + ACC;
   uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* redbar = drain + 1;        // cluster split-K: 2 barriers, alternating by unit
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
 
@@ -242,6 +335,10 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       ptx::mbar_init(ptx::smem_u32(&tempty[a]), 128);
     }
     ptx::mbar_init(ptx::smem_u32(drain), 1);
+    if (p.cluster > 0) {
+      ptx::mbar_init(ptx::smem_u32(&redbar[0]), uint32_t(p.cluster));
+      ptx::mbar_init(ptx::smem_u32(&redbar[1]), uint32_t(p.cluster));
+    }
     *abort_flag = 0;
     *last_flag = 0;
     ptx::fence_barrier_init();
@@ -254,6 +351,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  // peers signal this CTA's reduction barriers: every CTA of the cluster must
+  // have initialised them before any signal is sent
+  if (p.cluster > 0) ptx::cluster_sync_all();
   const uint32_t tmem_base = *tmem_slot;
   if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
@@ -369,8 +469,10 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     const int et = threadIdx.x - 64;        // 0 .. 127
     int acc = 0;
     uint32_t acc_phase = 0;
+    uint32_t red_it = 0;                    // cluster reductions done by this CTA
     for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
       const UnitCoord c = decode_unit(p, u);
+      bool released = false;                // accumulator already handed back
       bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
       ok = ptx::named_bar_and(1, 128, ok);
       if (!ok) {
@@ -414,6 +516,35 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
                             __uint_as_float(raw[4 * j4 + 2]), __uint_as_float(raw[4 * j4 + 3]));
         }
         __threadfence();
+        if (p.cluster > 0) {
+          // ---- cluster split-K: the S splits of this tile are the S CTAs of
+          // this cluster.  Publish the partial, signal every peer, wait for
+          // all S partials, then reduce this CTA's 1/S of the tile's rows.
+          ptx::tc_fence_before();
+          ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
+          released = true;
+          ptx::named_bar_sync(1, 128);
+          const uint32_t rb = ptx::smem_u32(&redbar[red_it & 1]);
+          if (et == 0) {
+            if (first_unit) trace_stamp(trace, kTrPartials);
+            for (int q2 = 0; q2 < w.split; ++q2) ptx::mbar_arrive_remote_release(ptx::map_to_rank(rb, uint32_t(q2)));
+          }
+          bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag);
+          ok2 = ptx::named_bar_and(1, 128, ok2);
+          ++red_it;
+          if (!ok2) {
+            if (et == 0) raise_error(p.err, abort_flag, kErrClusterWait);
+            break;
+          }
+          if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
+          const float4* tile_parts = part_base + size_t(c.tile * w.split) * TILE_F4;
+          switch (w.split) {
+            case 2: reduce_slice<MMA_N, 2, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
+            case 4: reduce_slice<MMA_N, 4, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
+            case 8: reduce_slice<MMA_N, 8, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
+            default: break;
+          }
+        } else {
         ptx::named_bar_sync(1, 128);
         if (et == 0) {
           if (first_unit) trace_stamp(trace, kTrPartials);
@@ -470,10 +601,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           }
           if (et == 0) w.ws_cnt[c.tile] = 0u;     // leave the counter zeroed for the next run
         }
+        }
       }
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstStore);
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));
+      if (!released) {
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));
+      }
       if (++acc == ACC) {
         acc = 0;
         acc_phase ^= 1;
@@ -490,6 +624,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       trace[blockIdx.x * kTracePerCta + kTrUnits] = n;
     }
   }
+  // no CTA of a cluster leaves while a peer may still signal its barriers
+  // (every role's waits are bounded, so every CTA gets here)
+  if (p.cluster > 0) ptx::cluster_sync_all();
   if (warp == 1) {
     __syncwarp();
     ptx::tc_fence_after();

@@ -53,6 +53,7 @@ struct DeviceState {
   int sm_count = 0;
   int* err_word = nullptr;
   int ctas_per_sm[kNumKinds][2][2] = {};   // [kind][bf16 out][fused]; 0 = not yet set up
+  int cluster_ok[kNumKinds][2][2][4] = {};  // [..][log2 cluster size]; 0 unknown, 1 yes, -1 no
 };
 
 std::mutex g_mu;
@@ -128,6 +129,59 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
   }
   *ctas = c;
   return GOLDY_OK;
+}
+
+// Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
+// cluster > 1.
+cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params, int cluster) {
+  void* args[] = {params};
+  if (cluster <= 1) return cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = unsigned(cluster);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
+// Can clusters of `cluster` CTAs of this kernel be resident at all?
+bool cluster_feasible(DeviceState& d, int kind, int out_bf16, int fused, int cluster) {
+  const int li = cluster == 2 ? 1 : cluster == 4 ? 2 : cluster == 8 ? 3 : 0;
+  if (li == 0) return false;
+  std::lock_guard<std::mutex> lock(g_mu);
+  int& c = d.cluster_ok[kind][out_bf16][fused][li];
+  if (c == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(cluster));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = size_t(smem_bytes(kKinds[kind]));
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = unsigned(cluster);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, kernel_fn(kind, out_bf16, fused), &cfg);
+    c = (e == cudaSuccess && n > 0) ? 1 : -1;
+    if (e != cudaSuccess) cudaGetLastError();     // clear; fall back to the unclustered reduction
+  }
+  return c > 0;
+}
+
+// Grid of a launch: the persistent cap, and a whole number of clusters.
+unsigned launch_grid(int64_t units, int64_t cap, int cluster) {
+  int64_t g = std::min<int64_t>(units, cap);
+  if (cluster > 1) g = std::max<int64_t>(cluster, (g / cluster) * cluster);
+  return unsigned(g);
 }
 
 goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
@@ -213,11 +267,11 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
 
   const Variant v = variant_of(gp.variant);
   const int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
-  const unsigned grid = unsigned(std::min<int64_t>(gp.units, cap));
+  const int cluster = (gp.split > 1 && cluster_feasible(d, gp.kind, out_bf16, 0, gp.split)) ? gp.split : 0;
+  p.cluster = cluster;
+  const unsigned grid = launch_grid(gp.units, cap, cluster);
   p.trace = trace_for(grid);
-  void* args[] = {&p};
-  cudaError_t e = cudaLaunchKernel(kernel_fn(gp.kind, out_bf16, 0), dim3(grid), dim3(kThreads), args,
-                                   size_t(smem_bytes(k)), stream);
+  cudaError_t e = launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, cluster);
   if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel");
   return GOLDY_OK;
 }
@@ -250,11 +304,15 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.total_units = int32_t(units);
   p.err = d.err_word;
   cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
-  const unsigned grid = unsigned(std::min<int64_t>(units, cap));
+  // clusters need one split factor for every GEMM of the launch
+  int split = g0.split;
+  for (int j = 1; j < count; ++j)
+    if (s->gemms[members[j]].split != split) split = 0;
+  const int cluster = (split > 1 && cluster_feasible(d, g0.kind, out_bf16, 1, split)) ? split : 0;
+  p.cluster = cluster;
+  const unsigned grid = launch_grid(units, cap, cluster);
   p.trace = trace_for(grid);
-  void* args[] = {&p};
-  cudaError_t e = cudaLaunchKernel(kernel_fn(g0.kind, out_bf16, 1), dim3(grid), dim3(kThreads), args,
-                                   size_t(smem_bytes(k)), stream);
+  cudaError_t e = launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, cluster);
   if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (fused)");
   return GOLDY_OK;
 }
