@@ -110,7 +110,8 @@ const char* goldy_last_error(void);
  * A variant is one GO-Kernel configuration (Sec. 4.2): a tile shape and
  * shared-memory/tensor-memory footprint (kind), a split of the K loop, and a
  * resource constraint (RC) capping the persistent grid at the whole GPU, half
- * or a quarter of it (Sec. 4.2.1's GPU, GPU/2, GPU/4). */
+ * or a quarter of it (Sec. 4.2.1's GPU, GPU/2, GPU/4).  Kinds whose tiles are
+ * computed by a CTA pair ignore the split factor (they never split K). */
 typedef struct goldy_variant_info {
   int32_t id;
   int32_t kind;           /* tile/footprint family, 0 .. n_kinds-1 */
@@ -124,6 +125,8 @@ typedef struct goldy_variant_info {
   int32_t split_k;        /* K-loop split factor (1, 2, 4, 8) */
   int32_t rc_div;         /* grid cap = resident CTAs per SM * SMs / rc_div */
   int32_t ctas_per_sm;    /* CTAs per SM the footprint is sized for */
+  int32_t cta_pair;       /* 2: tiles of 2 x 128 rows computed by a pair of CTAs
+                             (one tcgen05 MMA across both SMs), else 1 */
   char name[32];
 } goldy_variant_info;
 

@@ -23,7 +23,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libgoldy.so")
-NUM_KINDS = 10
+NUM_KINDS = 11
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

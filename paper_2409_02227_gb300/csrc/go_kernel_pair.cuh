@@ -1,0 +1,267 @@
+// GO-Kernel over CTA pairs: 256 x 256 output tiles with tcgen05.mma.cta_group::2.
+//
+// Same GEMM as go_gemm_kernel (Sec. 2.1.2, C = A * B, fp32 accumulation), for
+// compute-bound shapes.  A cluster of two CTAs on neighbouring SMs works on one
+// 256 x 256 tile at a time: CTA r (r = 0, 1) loads rows 128r .. 128r+127 of the
+// tile's A panel and columns 128r .. 128r+127 of its B panel into its own
+// shared memory, the even CTA issues one 256 x 256 x 16 MMA per K step that
+// reads both CTAs' operands, and each CTA's tensor memory receives its 128
+// rows of the accumulator.  Per K block each SM therefore takes in 32 KB of
+// operands for 128 x 256 x 64 multiply-adds — two thirds of what the
+// single-CTA 128 x 256 tile needs — which keeps the tensor cores fed from L2.
+//
+// Roles per CTA (192 threads): warp 0 lane 0 loads (both CTAs; the odd CTA's
+// loads complete on the even CTA's barrier), warp 1 allocates tensor memory
+// jointly with the peer and, in the even CTA, issues the MMAs and commits
+// (multicast to both CTAs' barriers), warps 2-5 drain the CTA's own half of
+// the accumulator.  Units (256 x 256 tiles) go to pairs round-robin; both CTAs
+// of a pair walk the same sequence.  Every wait is bounded; before leaving,
+// each CTA waits (bounded) until every arrival the peer owes its barriers has
+// landed, then the pair meets at a cluster barrier.
+#pragma once
+
+#include "go_kernel.cuh"
+
+namespace goldy {
+
+template <bool OUT_BF16, int MAXG>
+__global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_constant__ LaunchParams<MAXG> p) {
+  constexpr int STAGES = 6;
+  constexpr int ACC = 2;
+  constexpr int HALF_N = 128;                        // B columns held per CTA
+  constexpr int A_BYTES = 128 * 64 * 2;              // 128 rows of A x 64 K
+  constexpr int B_BYTES = HALF_N * 64 * 2;           // 128 columns of B x 64 K
+  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr uint32_t TMEM_COLS = 512;                // 2 accumulators x 256 fp32 columns
+  constexpr uint32_t IDESC = ptx::make_idesc_bf16(256, 256, 0, 1);
+  constexpr uint32_t KMAJ_STEP = 32;
+  constexpr uint32_t MNMAJ_STEP = 2048;
+  constexpr uint32_t MNMAJ_LBO = 64 * 128;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* full = bars;                    // used in the even CTA: both CTAs' loads complete here
+  uint64_t* empty = bars + STAGES;          // each CTA: its slot was consumed by the pair MMA
+  uint64_t* tfull = bars + 2 * STAGES;      // each CTA: its half of the accumulator is ready
+  uint64_t* tempty = bars + 2 * STAGES + ACC;  // even CTA: both halves were drained (2 arrivals)
+  uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const uint32_t tiles_base = ptx::smem_u32(smem);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = ptx::cluster_ctarank() & 1u;
+  const bool lead = rank == 0;
+  const int pair = blockIdx.x >> 1;
+  const int n_pairs = gridDim.x >> 1;
+  unsigned long long* const trace = p.trace;
+
+  if (threadIdx.x == 0) {
+    trace_stamp(trace, kTrStart);
+    if (trace) {
+      uint32_t sm;
+      asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+      trace[blockIdx.x * kTracePerCta + kTrSm] = sm;
+    }
+    for (int g = 0; g < p.n_gemms; ++g) {
+      ptx::prefetch_tensormap(&p.tmap_a[g]);
+      ptx::prefetch_tensormap(&p.tmap_b[g]);
+    }
+    for (int s = 0; s < STAGES; ++s) {
+      ptx::mbar_init(ptx::smem_u32(&full[s]), 1);
+      ptx::mbar_init(ptx::smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < ACC; ++a) {
+      ptx::mbar_init(ptx::smem_u32(&tfull[a]), 1);
+      ptx::mbar_init(ptx::smem_u32(&tempty[a]), 2);
+    }
+    ptx::mbar_init(ptx::smem_u32(drain), 1);
+    *abort_flag = 0;
+    ptx::fence_barrier_init();
+    ptx::fence_proxy_async_smem();
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc_pair(ptx::smem_u32(tmem_slot), TMEM_COLS);
+    ptx::tmem_relinquish_pair();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  ptx::cluster_sync_all();                  // the peer's barriers and tensor memory are ready
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ producer
+      int stage = 0;
+      uint32_t phase = 0, issued = 0, last_phase = 0;
+      bool ok = true;
+      for (int u = pair; ok && u < p.total_units; u += n_pairs) {
+        const UnitCoord c = decode_unit(p, u);
+        const void* ta = &p.tmap_a[c.g];
+        const void* tb = &p.tmap_b[c.g];
+        const int m0 = c.tm * 256 + int(rank) * 128;
+        const int n0 = c.tn * 256 + int(rank) * HALF_N;
+        for (int kb = c.kb0; kb < c.kb1; ++kb) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb_local = ptx::smem_u32(&full[stage]);
+          const uint32_t fb = ptx::map_to_rank(fb_local, 0);      // the even CTA's barrier
+          if (lead) ptx::mbar_arrive_expect_tx(fb_local, 2 * STAGE_BYTES);
+          const uint32_t xs = tiles_base + stage * STAGE_BYTES;
+          const uint32_t ys = xs + A_BYTES;
+          const int k0 = kb * 64;
+          ptx::tma_load_2d_pair(xs, ta, fb, k0, m0);
+          ptx::tma_load_2d_pair(ys, tb, fb, n0, k0);
+          ptx::tma_load_2d_pair(ys + 8192, tb, fb, n0 + 64, k0);
+          if (issued == 0) trace_stamp(trace, kTrFirstLoad);
+          issued |= 1u << stage;
+          last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (!ok) raise_error(p.err, abort_flag, kErrProducerWait);
+      // every slot this CTA filled must have been released by the pair MMA
+      // (so the even CTA's commits to this CTA's barriers have landed, and
+      // the peer's loads into the even CTA's slots are done) before leaving
+      const uint64_t t0 = ptx::global_timer();
+      for (int s = 0; s < STAGES; ++s) {
+        if (!(issued >> s & 1)) continue;
+        const uint32_t bar = ptx::smem_u32(&empty[s]);
+        const uint32_t par = (last_phase >> s) & 1;
+        while (!ptx::mbar_try_wait(bar, par)) {
+          if (ptx::global_timer() - t0 > ptx::kWaitLimitNs) {
+            raise_error(p.err, abort_flag, kErrProducerWait);
+            break;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && lead) {
+      // ------------------------------------------------- MMA issuer (even CTA)
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true, any = false;
+      for (int u = pair; ok && u < p.total_units; u += n_pairs) {
+        const UnitCoord c = decode_unit(p, u);
+        // both CTAs drained this accumulator (the odd CTA signals with a
+        // cluster-scope release, so wait with a cluster-scope acquire)
+        if (!ptx::mbar_wait_cluster(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + uint32_t(acc * 256);
+        for (int kb = c.kb0; kb < c.kb1; ++kb) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          if (!any) trace_stamp(trace, kTrFirstFull);
+          const uint32_t xs = tiles_base + stage * STAGE_BYTES;
+          const uint32_t ys = xs + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t adesc = ptx::make_sdesc_sw128(xs + kk * KMAJ_STEP, 16, 1024);
+            const uint64_t bdesc = ptx::make_sdesc_sw128(ys + kk * MNMAJ_STEP, MNMAJ_LBO, 1024);
+            ptx::mma_bf16_pair(d_tmem, adesc, bdesc, IDESC, (kb > c.kb0 || kk > 0) ? 1u : 0u);
+          }
+          any = true;
+          ptx::mma_commit_pair_multicast(ptx::smem_u32(&empty[stage]), 0x3);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        ptx::mma_commit_pair_multicast(ptx::smem_u32(&tfull[acc]), 0x3);
+        if (u == pair) trace_stamp(trace, kTrFirstMmaDone);
+        if (++acc == ACC) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
+      }
+      if (!ok) {
+        raise_error(p.err, abort_flag, kErrMmaWait);
+        if (any) {
+          ptx::mma_commit_pair_multicast(ptx::smem_u32(drain), 0x1);
+          ptx::mbar_wait(ptx::smem_u32(drain), 0, nullptr);
+        }
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const int et = threadIdx.x - 64;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int u = pair; u < p.total_units; u += n_pairs) {
+      const UnitCoord c = decode_unit(p, u);
+      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
+      ok = ptx::named_bar_and(1, 128, ok);
+      if (!ok) {
+        if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
+        break;
+      }
+      ptx::tc_fence_after();
+      const bool first_unit = (u == pair);
+      if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
+      const GemmWork& w = p.g[c.g];
+      const int m0 = c.tm * 256 + int(rank) * 128;
+      const int n0 = c.tn * 256;
+      const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
+#pragma unroll 1
+      for (int c0 = 0; c0 < 256; c0 += 32) {
+        uint32_t raw[32];
+        __syncwarp();
+        ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+        ptx::tmem_ld_wait();
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
+        store_chunk<false, OUT_BF16>(w, m0, n0, r, c0, v);
+      }
+      if (first_unit && et == 0) trace_stamp(trace, kTrFirstStore);
+      ptx::tc_fence_before();
+      ptx::named_bar_sync(1, 128);
+      if (et == 0) {
+        // this CTA's half of accumulator `acc` is drained: tell the MMA issuer
+        ptx::mbar_arrive_remote_release(ptx::map_to_rank(ptx::smem_u32(&tempty[acc]), 0));
+      }
+      if (++acc == ACC) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+  }
+
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    trace_stamp(trace, kTrEnd);
+    if (trace) {
+      int n = 0;
+      for (int u = pair; u < p.total_units; u += n_pairs) ++n;
+      trace[blockIdx.x * kTracePerCta + kTrUnits] = n;
+    }
+  }
+  ptx::cluster_sync_all();                  // no CTA of the pair leaves while the other may still signal it
+  if (warp == 1) {
+    __syncwarp();
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace goldy

@@ -30,9 +30,10 @@ struct KindInfo {
   int stages;      // shared-memory pipeline stages
   int acc_stages;  // accumulators in tensor memory (double buffering across tiles)
   int ctas_per_sm; // footprint target
+  int pair;        // 1: a cluster of two CTAs computes 256-row tiles with one MMA (cta_group::2)
 };
 
-constexpr int kNumKinds = 10;
+constexpr int kNumKinds = 11;
 constexpr int kMmaM = 128;          // rows of every tensor-core tile
 constexpr int kBlockK = 64;         // K elements per pipeline stage (one 128-byte row of bf16)
 constexpr int kSplits[4] = {1, 2, 4, 8};
@@ -41,21 +42,23 @@ constexpr int kNumVariants = kNumKinds * 4 * 3;
 constexpr int kThreads = 192;       // 1 TMA warp, 1 MMA warp, 4 epilogue warps
 
 inline constexpr KindInfo kKinds[kNumKinds] = {
-    // name        mma_n swap stages acc ctas/SM
-    {"n64_full", 64, 0, 8, 2, 1},
-    {"n64_half", 64, 0, 4, 2, 2},
-    {"n128_full", 128, 0, 6, 2, 1},
-    {"n128_half", 128, 0, 3, 2, 2},
-    {"n256_full", 256, 0, 4, 2, 1},
-    {"n256_half", 256, 0, 2, 1, 2},
-    {"t32_full", 32, 1, 8, 2, 1},
-    {"t32_half", 32, 1, 4, 2, 2},
-    {"t64_full", 64, 1, 8, 2, 1},
-    {"t64_half", 64, 1, 4, 2, 2},
+    // name        mma_n swap stages acc ctas/SM pair
+    {"n64_full", 64, 0, 8, 2, 1, 0},
+    {"n64_half", 64, 0, 4, 2, 2, 0},
+    {"n128_full", 128, 0, 6, 2, 1, 0},
+    {"n128_half", 128, 0, 3, 2, 2, 0},
+    {"n256_full", 256, 0, 4, 2, 1, 0},
+    {"n256_half", 256, 0, 2, 1, 2, 0},
+    {"t32_full", 32, 1, 8, 2, 1, 0},
+    {"t32_half", 32, 1, 4, 2, 2, 0},
+    {"t64_full", 64, 1, 8, 2, 1, 0},
+    {"t64_half", 64, 1, 4, 2, 2, 0},
+    {"p256_pair", 256, 0, 6, 2, 1, 1},   // 256 x 256 tiles over a CTA pair; split-K is not used
 };
 
 constexpr int stage_bytes(const KindInfo& k) {
-  return kMmaM * kBlockK * 2 + k.mma_n * kBlockK * 2;
+  // a CTA of a pair holds 128 rows of A and half of the tile's B columns
+  return kMmaM * kBlockK * 2 + (k.pair ? k.mma_n / 2 : k.mma_n) * kBlockK * 2;
 }
 constexpr int tmem_cols(const KindInfo& k) {
   int c = k.mma_n * k.acc_stages;
@@ -82,8 +85,10 @@ inline int variant_id(int kind, int split_idx, int rc_idx) { return (kind * 4 + 
 // Tile grid of one GEMM under a kind: the output is cut into tiles of
 // (tile_m x tile_n) elements of C.
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
-inline int tile_rows(const KindInfo& k) { return k.swap_ab ? k.mma_n : kMmaM; }
+inline int tile_rows(const KindInfo& k) { return k.pair ? 2 * kMmaM : (k.swap_ab ? k.mma_n : kMmaM); }
 inline int tile_cols(const KindInfo& k) { return k.swap_ab ? kMmaM : k.mma_n; }
+// rows of A one CTA loads per K block (the TMA box height)
+inline int a_box_rows(const KindInfo& k) { return k.pair ? kMmaM : tile_rows(k); }
 
 // ---------------------------------------------------------------------------
 // Schedule
@@ -124,6 +129,7 @@ const void* kernel_fn_k6(int out_bf16, int fused);
 const void* kernel_fn_k7(int out_bf16, int fused);
 const void* kernel_fn_k8(int out_bf16, int fused);
 const void* kernel_fn_k9(int out_bf16, int fused);
+const void* kernel_fn_k10(int out_bf16, int fused);
 
 }  // namespace goldy
 

@@ -3,6 +3,7 @@
 // forms (one GEMM per launch, or up to kMaxFused GEMMs).  One object per kind
 // keeps the build parallel.
 #include "go_kernel.cuh"
+#include "go_kernel_pair.cuh"
 #include "goldy_internal.h"
 
 #ifndef GOLDY_KIND
@@ -14,22 +15,35 @@
 
 namespace goldy {
 
-namespace {
-constexpr KindInfo kK = kKinds[GOLDY_KIND];
-constexpr bool kSwap = kK.swap_ab != 0;
-}  // namespace
-
-const void* GOLDY_CAT(kernel_fn_k, GOLDY_KIND)(int out_bf16, int fused) {
-  if (fused) {
+// Inside a template, `if constexpr` discards the other family entirely.
+template <int KIND>
+const void* select_kernel(int out_bf16, int fused) {
+  constexpr KindInfo k = kKinds[KIND];
+  constexpr bool swap = k.swap_ab != 0;
+  if constexpr (k.pair != 0) {
+    if (fused)
+      return out_bf16 ? reinterpret_cast<const void*>(&go_gemm_pair_kernel<true, kMaxFused>)
+                      : reinterpret_cast<const void*>(&go_gemm_pair_kernel<false, kMaxFused>);
+    return out_bf16 ? reinterpret_cast<const void*>(&go_gemm_pair_kernel<true, 1>)
+                    : reinterpret_cast<const void*>(&go_gemm_pair_kernel<false, 1>);
+  } else {
+    if (fused) {
+      if (out_bf16)
+        return reinterpret_cast<const void*>(
+            &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, kMaxFused, k.ctas_per_sm>);
+      return reinterpret_cast<const void*>(
+          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, kMaxFused, k.ctas_per_sm>);
+    }
     if (out_bf16)
       return reinterpret_cast<const void*>(
-          &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, kMaxFused, kK.ctas_per_sm>);
+          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, 1, k.ctas_per_sm>);
     return reinterpret_cast<const void*>(
-        &go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, kMaxFused, kK.ctas_per_sm>);
+        &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, 1, k.ctas_per_sm>);
   }
-  if (out_bf16)
-    return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, true, 1, kK.ctas_per_sm>);
-  return reinterpret_cast<const void*>(&go_gemm_kernel<kK.mma_n, kSwap, kK.stages, kK.acc_stages, false, 1, kK.ctas_per_sm>);
+}
+
+const void* GOLDY_CAT(kernel_fn_k, GOLDY_KIND)(int out_bf16, int fused) {
+  return select_kernel<GOLDY_KIND>(out_bf16, fused);
 }
 
 }  // namespace goldy

@@ -91,7 +91,7 @@ extern "C" goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int vari
   gp.tiles_m = ceil_div(desc->M, tile_rows(k));
   gp.tiles_n = ceil_div(desc->N, tile_cols(k));
   gp.k_blocks = ceil_div(desc->K, kBlockK);
-  gp.split = int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
+  gp.split = k.pair ? 1 : int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
   const int64_t tiles = gp.tiles_m * gp.tiles_n;
   gp.units = desc->K > 0 ? tiles * gp.split : 0;
   size_t need = 0, cnt_off = 0;

@@ -205,7 +205,7 @@ void finalize_schedule(goldy_schedule* s) {
     gp.tiles_m = ceil_div(gp.desc.M, tile_rows(k));
     gp.tiles_n = ceil_div(gp.desc.N, tile_cols(k));
     gp.k_blocks = ceil_div(gp.desc.K, kBlockK);
-    gp.split = int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
+    gp.split = k.pair ? 1 : int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
     const int64_t tiles = gp.tiles_m * gp.tiles_n;
     gp.units = (gp.desc.K > 0) ? tiles * gp.split : 0;
     gp.ws_part_off = gp.ws_cnt_off = gp.ws_bytes = 0;
@@ -451,16 +451,17 @@ extern "C" goldy_status goldy_variant_info_get(int id, goldy_variant_info* out) 
   std::memset(out, 0, sizeof(*out));
   out->id = id;
   out->kind = v.kind;
-  out->mma_m = kMmaM;
+  out->mma_m = k.pair ? 2 * kMmaM : kMmaM;
   out->mma_n = k.mma_n;
   out->swap_ab = k.swap_ab;
   out->stages = k.stages;
   out->acc_stages = k.acc_stages;
   out->tmem_cols = tmem_cols(k);
   out->smem_bytes = smem_bytes(k);
-  out->split_k = v.split;
+  out->split_k = k.pair ? 1 : v.split;
   out->rc_div = v.rc_div;
   out->ctas_per_sm = k.ctas_per_sm;
+  out->cta_pair = k.pair ? 2 : 1;
   std::snprintf(out->name, sizeof(out->name), "%s_s%d_rc%d", k.name, v.split, v.rc_div);
   return ok();
 }

@@ -76,6 +76,7 @@ const void* kernel_fn(int kind, int out_bf16, int fused) {
     case 7: return kernel_fn_k7(out_bf16, fused);
     case 8: return kernel_fn_k8(out_bf16, fused);
     case 9: return kernel_fn_k9(out_bf16, fused);
+    case 10: return kernel_fn_k10(out_bf16, fused);
     default: return nullptr;
   }
 }
@@ -184,6 +185,12 @@ unsigned launch_grid(int64_t units, int64_t cap, int cluster) {
   return unsigned(g);
 }
 
+// Pair kinds: every unit (a 256-row tile) occupies a cluster of two CTAs.
+unsigned pair_grid(int64_t units, int64_t cap) {
+  const int64_t pairs = std::max<int64_t>(1, std::min<int64_t>(units, cap / 2));
+  return unsigned(2 * pairs);
+}
+
 goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                        uint32_t box_inner, uint32_t box_outer) {
   cuuint64_t dims[2] = {inner, outer};
@@ -206,7 +213,7 @@ goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const v
   const goldy_gemm_desc& g = gp.desc;
   const KindInfo& k = kKinds[gp.kind];
   goldy_status st =
-      encode_2d(&p.tmap_a[j], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(tile_rows(k)));
+      encode_2d(&p.tmap_a[j], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(a_box_rows(k)));
   if (st != GOLDY_OK) return st;
   st = encode_2d(&p.tmap_b[j], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.ldb) * 2, 64, kBlockK);
   if (st != GOLDY_OK) return st;
@@ -267,6 +274,13 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
 
   const Variant v = variant_of(gp.variant);
   const int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
+  if (k.pair) {
+    const unsigned grid = pair_grid(gp.units, cap);
+    p.trace = trace_for(grid);
+    cudaError_t e = launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, 2);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (pair)");
+    return GOLDY_OK;
+  }
   const int cluster = (gp.split > 1 && cluster_feasible(d, gp.kind, out_bf16, 0, gp.split)) ? gp.split : 0;
   p.cluster = cluster;
   const unsigned grid = launch_grid(gp.units, cap, cluster);
@@ -304,6 +318,13 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.total_units = int32_t(units);
   p.err = d.err_word;
   cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
+  if (k.pair) {
+    const unsigned grid = pair_grid(units, cap);
+    p.trace = trace_for(grid);
+    cudaError_t e = launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, 2);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (fused pair)");
+    return GOLDY_OK;
+  }
   // clusters need one split factor for every GEMM of the launch
   int split = g0.split;
   for (int j = 1; j < count; ++j)

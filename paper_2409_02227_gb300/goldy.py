@@ -65,7 +65,7 @@ class goldy_run_opts(ctypes.Structure):
 class goldy_variant_info(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("id", "kind", "mma_m", "mma_n", "swap_ab", "stages", "acc_stages", "tmem_cols",
-                 "smem_bytes", "split_k", "rc_div", "ctas_per_sm")] + [("name", ctypes.c_char * 32)]
+                 "smem_bytes", "split_k", "rc_div", "ctas_per_sm", "cta_pair")] + [("name", ctypes.c_char * 32)]
 
     def as_dict(self) -> dict:
         d = {n: getattr(self, n) for n, _ in self._fields_ if n != "name"}

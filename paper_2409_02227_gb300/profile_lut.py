@@ -52,6 +52,7 @@ RC_DIVS = (1, 2, 4)
 SPLITS = (1, 2, 4, 8)
 SWAP_KINDS = (6, 7, 8, 9)
 NONSWAP_KINDS = (0, 1, 2, 3, 4, 5)
+PAIR_KINDS = (10,)
 
 
 def write_lut(entries: Sequence[Tuple[Tuple[int, int, int, int], int, Sequence[int]]],
@@ -86,16 +87,17 @@ def bucket_shape(key) -> Tuple[int, int, int, int]:
 
 
 def candidates(M: int, N: int, K: int, sm_count: int) -> List[Tuple[int, int]]:
-    kinds = list(NONSWAP_KINDS) + (list(SWAP_KINDS) if M <= 128 else [])
+    kinds = (list(NONSWAP_KINDS) + (list(SWAP_KINDS) if M <= 128 else [])
+             + (list(PAIR_KINDS) if M > 128 else []))
     k_blocks = math.ceil(K / 64)
     out = []
     for kind in kinds:
         info = G.goldy_variant_info_get(G.variant_id(kind, 1, 1))
-        rows = info["mma_n"] if info["swap_ab"] else 128
+        rows = info["mma_n"] if info["swap_ab"] else info["mma_m"]
         cols = 128 if info["swap_ab"] else info["mma_n"]
         tiles = math.ceil(M / rows) * math.ceil(N / cols)
         for s in SPLITS:
-            if s > 1 and (s > k_blocks or tiles * s > 4 * sm_count):
+            if s > 1 and (info["cta_pair"] == 2 or s > k_blocks or tiles * s > 4 * sm_count):
                 continue
             out.append((kind, s))
     return out

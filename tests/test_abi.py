@@ -34,12 +34,14 @@ def test_every_declared_symbol_is_exported():
 def test_version_and_registry():
     assert G.goldy_abi_version() == 1
     n = G.goldy_variant_count()
-    assert n == 120
+    assert n == 132
     seen = set()
     for v in range(n):
         info = G.goldy_variant_info_get(v)
-        assert info["id"] == v and info["mma_m"] == 128
+        assert info["id"] == v and info["mma_m"] == 128 * info["cta_pair"]
         assert info["split_k"] in (1, 2, 4, 8) and info["rc_div"] in (1, 2, 4)
+        if info["cta_pair"] == 2:
+            assert info["split_k"] == 1
         assert info["tmem_cols"] in (32, 64, 128, 256, 512)
         assert info["tmem_cols"] >= info["mma_n"] * info["acc_stages"]
         # footprint: "half" kinds leave room for a second CTA on the SM
@@ -47,7 +49,7 @@ def test_version_and_registry():
             assert info["smem_bytes"] <= 113 * 1024 and info["tmem_cols"] <= 256
         assert info["smem_bytes"] <= 227 * 1024
         seen.add((info["kind"], info["split_k"], info["rc_div"]))
-    assert len(seen) == n
+    assert len(seen) == n - 12 + 3          # the pair kind reports split 1 for all its ids
     with pytest.raises(G.GoldyError) as e:
         G.goldy_variant_info_get(n)
     assert e.value.status == G.GOLDY_ERR_INVALID_ARG
@@ -108,7 +110,7 @@ def test_lut_error_paths(tmp_path):
         G.goldy_lut_load(str(tmp_path / "missing.bin"))
     assert e.value.status == G.GOLDY_ERR_LUT
     data = bytearray(_lut_bytes())
-    data[16] = 121                                            # variant bound beyond this library
+    data[16] = 133                                            # variant bound beyond this library
     with pytest.raises(G.GoldyError):
         G.goldy_lut_from_memory(bytes(data))
     p = tmp_path / "ok.bin"
@@ -131,7 +133,7 @@ def test_schedule_build_and_query():
     with pytest.raises(G.GoldyError):
         G.goldy_schedule_build(descs, [0, 2, 2], [0, 0, 0], [0, 0, 0])   # group 1 empty
     with pytest.raises(G.GoldyError):
-        G.goldy_schedule_build(descs, [0, 0, 0], [0, 0, 120], [0, 0, 0])
+        G.goldy_schedule_build(descs, [0, 0, 0], [0, 0, 132], [0, 0, 0])
     with pytest.raises(G.GoldyError):
         G.goldy_schedule_build(descs, [0, 0, 0], [0, 0, 0], [0, 0, 16])
     with pytest.raises(G.GoldyError):

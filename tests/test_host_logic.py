@@ -39,7 +39,9 @@ def test_bucket_shapes_and_candidates():
     kinds = {k for k, _ in c}
     assert {6, 7, 8, 9} <= kinds                      # transposed tiles offered for skinny M
     assert all(s in (1, 2, 4, 8) for _, s in c)
-    assert not {6, 7, 8, 9} & {k for k, _ in P.candidates(512, 1024, 1024, 152)}
+    big = {k for k, _ in P.candidates(512, 1024, 1024, 152)}
+    assert not {6, 7, 8, 9} & big and 10 in big
+    assert all(s == 1 for k, s in P.candidates(512, 1024, 1024, 152) if k == 10)
 
 
 def _free_port():
