@@ -332,13 +332,22 @@ def goldy_device_info(variant_id: int = 0) -> Tuple[int, int]:
     return sm.value, ctas.value
 
 
+_SPLITS = (1, 2, 4, 8)
+_RC_DIVS = (1, 2, 4)
+
+
 def variant_id(kind: int, split: int, rc_div: int) -> int:
-    """Variant id of (kind, split-K factor, grid-cap divisor), by registry lookup."""
-    for v in range(goldy_variant_count()):
-        info = goldy_variant_info_get(v)
-        if info["kind"] == kind and info["split_k"] == split and info["rc_div"] == rc_div:
-            return v
-    raise KeyError((kind, split, rc_div))
+    """Variant id of (kind, split-K factor, grid-cap divisor): the registry's
+    numbering (kind * 4 + split index) * 3 + RC index, checked against it."""
+    if split not in _SPLITS or rc_div not in _RC_DIVS:
+        raise KeyError((kind, split, rc_div))
+    v = (int(kind) * 4 + _SPLITS.index(split)) * 3 + _RC_DIVS.index(rc_div)
+    if not 0 <= v < goldy_variant_count():
+        raise KeyError((kind, split, rc_div))
+    info = goldy_variant_info_get(v)
+    if info["kind"] != kind or info["rc_div"] != rc_div or info["split_k"] not in (split, 1):
+        raise KeyError((kind, split, rc_div))
+    return v
 
 
 def kind_names() -> List[str]:
