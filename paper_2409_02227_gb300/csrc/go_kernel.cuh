@@ -52,13 +52,15 @@ struct GemmWork {
   int32_t split;        // K-range split, 1 <= split <= k_blocks
   int32_t k_blocks;     // ceil(K / 64)
   int32_t unit_begin;   // first unit of this GEMM within the launch
-  int32_t pad_[3];
+  int32_t c_tma;        // 1: C is written through tmap_c by TMA stores
+  int32_t pad_[2];
 };
 
 template <int MAXG>
 struct LaunchParams {
   CUtensorMap tmap_a[MAXG];   // A: dims {K, M}, box {64, rows of the A tile}
   CUtensorMap tmap_b[MAXG];   // B: dims {N, K}, box {64, 64}
+  CUtensorMap tmap_c[MAXG];   // C: dims {N, M}, box {128-byte row, 128 rows} (when g[].c_tma)
   GemmWork g[MAXG];
   int32_t n_gemms;
   int32_t total_units;
@@ -270,13 +272,72 @@ __device__ __forceinline__ void reduce_slice(const GemmWork& w, const float4* ti
   }
 }
 
+// Store one accumulator tile (128 rows x MMA_N columns, rows m0.., columns
+// n0..) through shared memory with TMA.  Per chunk of 128-byte rows (32 fp32
+// or 64 bf16 columns) every thread writes its row into a staging buffer with
+// the 128-byte swizzle (so a warp's writes hit distinct banks), then one
+// thread issues the tensor store; two 16 KB buffers alternate, and a buffer
+// is reused only after the store two chunks back has read it.  The store
+// clips rows and columns outside C.
+template <int MMA_N, bool OUT_BF16>
+__device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t staging, uint32_t& stg, uint32_t taddr,
+                                               int r, int et, int m0, int n0) {
+  constexpr int CHUNK = OUT_BF16 ? 64 : 32;
+#pragma unroll 1
+  for (int c0 = 0; c0 < MMA_N; c0 += CHUNK) {
+    const uint32_t buf = staging + (stg & 1u) * 16384u;
+    if (et == 0) ptx::bulk_wait_group_read<1>();
+    ptx::named_bar_sync(1, 128);
+    const uint32_t row = buf + uint32_t(r) * 128u;
+    const uint32_t sw = uint32_t(r & 7);
+    uint32_t raw[32];
+    __syncwarp();
+    ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+    ptx::tmem_ld_wait();
+    if (!OUT_BF16) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        ptx::st_shared_v4(row + ((uint32_t(j) ^ sw) << 4), raw[4 * j], raw[4 * j + 1], raw[4 * j + 2], raw[4 * j + 3]);
+    } else {
+      uint32_t pk[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(raw[2 * j]), __uint_as_float(raw[2 * j + 1]));
+        pk[j] = *reinterpret_cast<uint32_t*>(&h);
+      }
+      __syncwarp();
+      ptx::tmem_ld_32x32b_x32(taddr + c0 + 32, raw);
+      ptx::tmem_ld_wait();
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        ptx::st_shared_v4(row + ((uint32_t(j) ^ sw) << 4), pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(raw[2 * j]), __uint_as_float(raw[2 * j + 1]));
+        pk[j] = *reinterpret_cast<uint32_t*>(&h);
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        ptx::st_shared_v4(row + ((uint32_t(j + 4) ^ sw) << 4), pk[4 * j], pk[4 * j + 1], pk[4 * j + 2],
+                          pk[4 * j + 3]);
+    }
+    ptx::fence_proxy_async_smem();
+    ptx::named_bar_sync(1, 128);
+    if (et == 0) {
+      ptx::tma_store_2d(tmap_c, buf, n0 + c0, m0);
+      ptx::bulk_commit_group();
+    }
+    ++stg;
+  }
+}
+
 template <int MMA_N, int ACC>
 struct TmemCols {
   static constexpr uint32_t need = uint32_t(MMA_N * ACC);
   static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
 };
 
-template <int MMA_N, bool SWAP, int STAGES, int ACC, bool OUT_BF16, int MAXG, int MIN_CTAS>
+template <int MMA_N, bool SWAP, int STAGES, int ACC, bool OUT_BF16, int MAXG, int MIN_CTAS, bool EPI_TMA>
 __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_constant__ LaunchParams<MAXG> p) {
   constexpr int X_BYTES = 128 * 64 * 2;              // MMA operand A: 128 rows x 64 K
   constexpr int Y_BYTES = MMA_N * 64 * 2;            // MMA operand B: MMA_N rows x 64 K
@@ -294,10 +355,12 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   static_assert(MMA_N % 32 == 0 && MMA_N >= 32 && MMA_N <= 256, "MMA_N");
   static_assert(TILE_N % 64 == 0, "B tiles are whole 64-column boxes");
   static_assert(STAGES <= 32, "stage bitmasks");
+  static_assert(!(EPI_TMA && SWAP), "the TMA-store epilogue writes untransposed tiles");
+  constexpr int STAGING_BYTES = EPI_TMA ? 2 * 16384 : 0;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + STAGING_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* tfull = bars + 2 * STAGES;
@@ -470,6 +533,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     int acc = 0;
     uint32_t acc_phase = 0;
     uint32_t red_it = 0;                    // cluster reductions done by this CTA
+    uint32_t stg = 0;                       // staging buffers used (TMA-store epilogue)
+    const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
     for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
       const UnitCoord c = decode_unit(p, u);
       bool released = false;                // accumulator already handed back
@@ -486,7 +551,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);
-      if (w.split == 1) {
+      if (EPI_TMA && w.split == 1 && w.c_tma) {
+        store_tile_tma<MMA_N, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0);
+      } else if (w.split == 1) {
 #pragma unroll 1
         for (int c0 = 0; c0 < MMA_N; c0 += 32) {
           uint32_t raw[32];
@@ -613,6 +680,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         acc_phase ^= 1;
       }
     }
+    // tensor stores must have read the staging buffers before the CTA leaves
+    if (EPI_TMA && et == 0) ptx::bulk_wait_group<0>();
   }
 
   __syncthreads();

@@ -40,7 +40,8 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  constexpr int STAGING_BYTES = 2 * 16384;            // TMA-store epilogue buffers
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + STAGING_BYTES);
   uint64_t* full = bars;                    // used in the even CTA: both CTAs' loads complete here
   uint64_t* empty = bars + STAGES;          // each CTA: its slot was consumed by the pair MMA
   uint64_t* tfull = bars + 2 * STAGES;      // each CTA: its half of the accumulator is ready
@@ -68,6 +69,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     for (int g = 0; g < p.n_gemms; ++g) {
       ptx::prefetch_tensormap(&p.tmap_a[g]);
       ptx::prefetch_tensormap(&p.tmap_b[g]);
+      if (p.g[g].c_tma) ptx::prefetch_tensormap(&p.tmap_c[g]);
     }
     for (int s = 0; s < STAGES; ++s) {
       ptx::mbar_init(ptx::smem_u32(&full[s]), 1);
@@ -207,6 +209,8 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     const int et = threadIdx.x - 64;
     int acc = 0;
     uint32_t acc_phase = 0;
+    uint32_t stg = 0;
+    const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
     for (int u = pair; u < p.total_units; u += n_pairs) {
       const UnitCoord c = decode_unit(p, u);
       bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
@@ -222,16 +226,20 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       const int m0 = c.tm * 256 + int(rank) * 128;
       const int n0 = c.tn * 256;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
+      if (w.c_tma) {
+        store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0);
+      } else {
 #pragma unroll 1
-      for (int c0 = 0; c0 < 256; c0 += 32) {
-        uint32_t raw[32];
-        __syncwarp();
-        ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
-        ptx::tmem_ld_wait();
-        float v[32];
+        for (int c0 = 0; c0 < 256; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+          float v[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
-        store_chunk<false, OUT_BF16>(w, m0, n0, r, c0, v);
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
+          store_chunk<false, OUT_BF16>(w, m0, n0, r, c0, v);
+        }
       }
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstStore);
       ptx::tc_fence_before();
@@ -245,6 +253,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         acc_phase ^= 1;
       }
     }
+    if (et == 0) ptx::bulk_wait_group<0>();
   }
 
   __syncthreads();

@@ -66,8 +66,13 @@ constexpr int tmem_cols(const KindInfo& k) {
   while (p < c) p <<= 1;
   return p;
 }
-// stages, 1 KB for 1024-byte alignment of the swizzled tiles, 1 KB for barriers
-constexpr int smem_bytes(const KindInfo& k) { return k.stages * stage_bytes(k) + 2048; }
+// Kinds with a whole SM to themselves (and the pair kind) store C through
+// shared memory with TMA; they keep two 16 KB staging buffers.
+constexpr bool epi_tma(const KindInfo& k) { return k.pair || (!k.swap_ab && k.ctas_per_sm == 1); }
+// stages, staging, 1 KB for 1024-byte alignment of the swizzled tiles, 1 KB for barriers
+constexpr int smem_bytes(const KindInfo& k) {
+  return k.stages * stage_bytes(k) + (epi_tma(k) ? 2 * 16384 : 0) + 2048;
+}
 
 struct Variant {
   int id, kind, split, rc_div;

@@ -30,15 +30,15 @@ const void* select_kernel(int out_bf16, int fused) {
     if (fused) {
       if (out_bf16)
         return reinterpret_cast<const void*>(
-            &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, kMaxFused, k.ctas_per_sm>);
+            &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, kMaxFused, k.ctas_per_sm, epi_tma(k)>);
       return reinterpret_cast<const void*>(
-          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, kMaxFused, k.ctas_per_sm>);
+          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, kMaxFused, k.ctas_per_sm, epi_tma(k)>);
     }
     if (out_bf16)
       return reinterpret_cast<const void*>(
-          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, 1, k.ctas_per_sm>);
+          &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, true, 1, k.ctas_per_sm, epi_tma(k)>);
     return reinterpret_cast<const void*>(
-        &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, 1, k.ctas_per_sm>);
+        &go_gemm_kernel<k.mma_n, swap, k.stages, k.acc_stages, false, 1, k.ctas_per_sm, epi_tma(k)>);
   }
 }
 

@@ -192,12 +192,13 @@ unsigned pair_grid(int64_t units, int64_t cap) {
 }
 
 goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-                       uint32_t box_inner, uint32_t box_outer) {
+                       uint32_t box_inner, uint32_t box_outer,
+                       CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+  CUresult r = g_encode(m, dtype, 2, const_cast<void*>(ptr), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuTensorMapEncodeTiled failed with code " + std::to_string(int(r)));
@@ -228,6 +229,16 @@ goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const v
   w.split = gp.split;
   w.k_blocks = int32_t(gp.k_blocks);
   w.unit_begin = unit_begin;
+  // C through TMA stores: kinds that keep staging buffers, 16-byte aligned C
+  // and rows; the epilogue writes 128-byte rows (32 fp32 / 64 bf16 columns)
+  const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
+  w.c_tma = 0;
+  if (epi_tma(k) && gp.split == 1 && aligned(C, 16) && (size_t(g.ldc) * es) % 16 == 0) {
+    st = encode_2d(&p.tmap_c[j], C, uint64_t(g.N), uint64_t(g.M), uint64_t(g.ldc) * es, uint32_t(128 / es), 128,
+                   g.c_dtype == GOLDY_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+    if (st != GOLDY_OK) return st;
+    w.c_tma = 1;
+  }
   if (gp.split > 1) {
     w.ws_part = reinterpret_cast<float*>(ws + gp.ws_part_off);
     w.ws_cnt = reinterpret_cast<uint32_t*>(ws + gp.ws_cnt_off);
