@@ -265,10 +265,10 @@ unsigned long long* trace_for(unsigned grid) {
   return (t_trace && grid <= t_trace_ctas) ? t_trace : nullptr;
 }
 
-// share > 0: this launch gets that fraction of the GPU's CTA slots instead of
-// its variant's own grid cap (set for heterogeneous fused waves, see goldy_run_ex).
+// scale > 0: the launch's grid cap is its variant's cap times `scale` (set for
+// heterogeneous fused waves, see goldy_run_ex), at most the whole GPU.
 goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, const void* B, void* C, uint8_t* ws,
-                         cudaStream_t stream, double share = 0.0) {
+                         cudaStream_t stream, double scale = 0.0) {
   if (degenerate(gp)) return launch_degenerate(gp, C, stream);
   const KindInfo& k = kKinds[gp.kind];
   const int out_bf16 = gp.desc.c_dtype == GOLDY_BF16 ? 1 : 0;
@@ -286,8 +286,8 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   p.err = d.err_word;
 
   const Variant v = variant_of(gp.variant);
-  const int64_t cap = share > 0.0 ? std::max<int64_t>(2, int64_t(share * ctas * d.sm_count))
-                                  : std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
+  int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
+  if (scale > 0.0) cap = std::min<int64_t>(int64_t(ctas) * d.sm_count, int64_t(double(cap) * scale));
   if (k.pair) {
     const unsigned grid = pair_grid(gp.units, cap);
     p.trace = trace_for(grid);
@@ -310,7 +310,7 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
 // GPU.
 goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* members, int count,
                           const void* const* A, const void* const* B, void* const* C, uint8_t* ws,
-                          cudaStream_t stream, double share = 0.0) {
+                          cudaStream_t stream, double scale = 0.0) {
   const GemmPlan& g0 = s->gemms[members[0]];
   const KindInfo& k = kKinds[g0.kind];
   const int out_bf16 = g0.desc.c_dtype == GOLDY_BF16 ? 1 : 0;
@@ -331,8 +331,8 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.n_gemms = count;
   p.total_units = int32_t(units);
   p.err = d.err_word;
+  if (scale > 0.0) cap = int64_t(double(cap) * scale);
   cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
-  if (share > 0.0) cap = std::max<int64_t>(2, int64_t(share * ctas * d.sm_count));
   if (k.pair) {
     const unsigned grid = pair_grid(units, cap);
     p.trace = trace_for(grid);
@@ -442,7 +442,7 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
     // first of them.
     struct LaunchSet {
       int slot, n, degenerate, wave;
-      double share;
+      double scale;     // grid-cap scale for heterogeneous fused waves (0: none)
       int members[kMaxFused];
     };
     LaunchSet sets[GOLDY_MAX_GEMMS];
@@ -470,42 +470,28 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
           sets[target].n = 0;
           sets[target].degenerate = degenerate(gp) ? 1 : 0;
           sets[target].wave = w0;
-          sets[target].share = 0.0;
+          sets[target].scale = 0.0;
         }
         sets[target].members[sets[target].n++] = i;
       }
     }
-    // A fused wave whose launches are of different kinds runs those launches
-    // side by side.  Each GO-Kernel's grid cap was tuned among equal GEMMs;
-    // when the wave's launches together ask for more than the GPU, the GPU's
-    // CTA slots are divided among them in proportion to their FLOPs instead,
-    // so a large GEMM next to small ones is not held to the share it was
-    // given among its own kind.
+    // A fused wave whose GEMMs are of different kinds runs one launch per
+    // kind, side by side.  A GO-Kernel tuned for CD c was sized as one of c
+    // co-runners sharing the GPU; a launch that carries m of the wave's c
+    // GEMMs therefore gets c/m times its members' caps (at most the whole
+    // GPU).  Launches go out largest first, so smaller ones fill the SMs the
+    // larger one frees in its tail.
     if (fused) {
       for (int t0 = 0; t0 < n_sets;) {
-        int t1 = t0;
-        while (t1 < n_sets && sets[t1].wave == sets[t0].wave) ++t1;
-        int kernels = 0;
-        double want = 0.0, flops = 0.0;
-        for (int t = t0; t < t1; ++t) {
-          if (sets[t].degenerate) continue;
-          ++kernels;
-          for (int j = 0; j < sets[t].n; ++j) {
-            const GemmPlan& gp = s->gemms[sets[t].members[j]];
-            want += 1.0 / variant_of(gp.variant).rc_div;
-            flops += double(gp.desc.M) * double(gp.desc.N) * double(gp.desc.K);
-          }
+        int t1 = t0, kernels = 0, wave_size = 0;
+        while (t1 < n_sets && sets[t1].wave == sets[t0].wave) {
+          wave_size += sets[t1].n;
+          if (!sets[t1].degenerate) ++kernels;
+          ++t1;
         }
-        if (kernels > 1 && want > 1.0 && flops > 0.0)
-          for (int t = t0; t < t1; ++t) {
-            if (sets[t].degenerate) continue;
-            double f = 0.0;
-            for (int j = 0; j < sets[t].n; ++j) {
-              const GemmPlan& gp = s->gemms[sets[t].members[j]];
-              f += double(gp.desc.M) * double(gp.desc.N) * double(gp.desc.K);
-            }
-            sets[t].share = f / flops;
-          }
+        if (kernels > 1)
+          for (int t = t0; t < t1; ++t)
+            if (!sets[t].degenerate) sets[t].scale = double(wave_size) / double(sets[t].n);
         t0 = t1;
       }
     }
@@ -528,9 +514,9 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
       if (st != GOLDY_OK) return st;
       if (ls.n == 1) {
         const int i = ls.members[0];
-        st = launch_gemm(*d, s->gemms[i], A[i], B[i], C[i], ws, stream, ls.share);
+        st = launch_gemm(*d, s->gemms[i], A[i], B[i], C[i], ws, stream, ls.scale);
       } else {
-        st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream, ls.share);
+        st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream, ls.scale);
       }
       if (st != GOLDY_OK) return st;
       st = hook(opts ? opts->ev_end : nullptr, ls.members, ls.n, stream);
