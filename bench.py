@@ -56,6 +56,9 @@ def parse_args(argv=None):
                     help="fused: a wave's same-kind GEMMs share one launch; streams: one launch per GEMM")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--report", default=None, metavar="FILE",
+                    help="instead of the JSON line: time every fixed set and the 64 randomized sets "
+                         "under every policy and write a JSON report to FILE (markdown table on stdout)")
     return ap.parse_args(argv)
 
 
@@ -571,11 +574,90 @@ def run_gpu(args, world, rank, local):
     return 0
 
 
+def time_policies(st, lut, copies, steps):
+    """Makespan (us) of one set under each policy, timed like the main line."""
+    import torch
+    from paper_2409_02227_gb300 import goldy as G
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    out = {}
+    for name, flags in (("goldyloc", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED),
+                        ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
+                        ("sequential", G.GOLDY_PLAN_SEQUENTIAL),
+                        ("naive_streams", G.GOLDY_PLAN_DEFAULT),
+                        ("go_all_concurrent", G.GOLDY_PLAN_GO)):
+        sched = G.goldy_plan(descs, lut, flags)
+        r = SetRunner(st, sched, copies)
+        for k in range(10):
+            r.launch(k)
+        torch.cuda.synchronize()
+        out[name] = r.timed(steps)[0] / steps * 1e3
+        if name == "goldyloc":
+            out["plan"] = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
+        del r
+    if G.goldy_device_error(clear=True) != 0:
+        raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
+    return out
+
+
+def run_report(args, local):
+    """Every fixed set and the 64 randomized sets under every policy."""
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2409_02227_gb300 import goldy as G
+    from paper_2409_02227_gb300 import workloads as wl
+    lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    hbm, tf_burst, _, _ = peaks()
+    l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
+    rows = []
+    sets = [(n, wl.make_config(n)) for n in wl.FIXED_CONFIGS]
+    sets += [(f"sweep_{j:02d}", None) for j in range(wl.SWEEP_SETS)]
+    for name, st in sets:
+        if st is None:
+            st = wl.make_sweep_set(int(name.split("_")[1]))
+        in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
+        copies = max(2, math.ceil(2 * l2 / in_bytes))
+        steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
+        t = time_policies(st, lut, copies, steps)
+        if name in wl.FIXED_CONFIGS:
+            t["cublas_sequential_reference"] = cublas_reference_ms(st, copies, steps) * 1e3
+        roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
+        row = {"set": name, "n_gemms": len(st.specs), "flops": st.flops, "bytes": st.bytes,
+               "bound": "tensor" if st.flops / st.bytes > tf_burst * 1e12 / (hbm * 1e9) else "hbm",
+               "roof_us": roof_us, "us": {k: v for k, v in t.items() if k != "plan"},
+               "tflops": st.flops / (t["goldyloc"] * 1e-6) / 1e12,
+               "roofline_frac": roof_us / t["goldyloc"],
+               "speedup_vs_sequential": t["sequential"] / t["goldyloc"],
+               "speedup_vs_naive_streams": t["naive_streams"] / t["goldyloc"],
+               "plan": [{"group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl, "cd": cd}
+                        for g, v, sl, cd in t["plan"]]}
+        rows.append(row)
+        print(f"| {name} | {len(st.specs)} | {row['bound']} | {roof_us:.2f} | {t['goldyloc']:.2f} | "
+              f"{row['tflops']:.1f} | {row['roofline_frac']:.3f} | {row['speedup_vs_sequential']:.2f} | "
+              f"{row['speedup_vs_naive_streams']:.2f} |", flush=True)
+        del st
+        torch.cuda.empty_cache()
+    sweep = [r for r in rows if r["set"].startswith("sweep")]
+    geo = lambda xs: math.exp(sum(math.log(x) for x in xs) / len(xs))
+    summary = {"sweep_geomean_speedup_vs_sequential": geo([r["speedup_vs_sequential"] for r in sweep]),
+               "sweep_geomean_speedup_vs_naive_streams": geo([r["speedup_vs_naive_streams"] for r in sweep]),
+               "sweep_geomean_roofline_frac": geo([r["roofline_frac"] for r in sweep]),
+               "sweep_geomean_roofline_frac_tensor_bound": geo([r["roofline_frac"] for r in sweep
+                                                                if r["bound"] == "tensor"] or [1.0]),
+               "sweep_sets_faster_than_sequential": sum(r["speedup_vs_sequential"] > 1 for r in sweep),
+               "sweep_sets_faster_than_naive_streams": sum(r["speedup_vs_naive_streams"] > 1 for r in sweep)}
+    print(json.dumps(summary), flush=True)
+    with open(args.report, "w") as f:
+        json.dump({"rows": rows, "summary": summary, "peaks": {"hbm_gbs": hbm, "bf16_tflops": tf_burst}}, f, indent=1)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     world, rank, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, world, rank)
+    if args.report:
+        return run_report(args, local)
     return run_gpu(args, world, rank, local)
 
 

@@ -278,3 +278,19 @@ def test_phase_trace_is_consistent(cuda_ok):
     for r in rows.tolist():
         assert r[0] <= r[1] <= r[2] and r[1] <= r[3] <= r[4] and r[5] <= r[8] <= r[9]
         assert r[6] <= r[7] and r[4] <= r[5]
+
+
+@pytest.mark.parametrize("j", [0, 17, 63])
+def test_sweep_sets_through_the_planner(cuda_ok, j):
+    # randomized sets (2-16 GEMMs, M 16-4096, N, K 256-8192) through the
+    # packaged table in fused mode; sampled rows of every GEMM vs the oracle
+    st = wl.make_sweep_set(j)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    sched = G.goldy_plan(descs, G.goldy_lut_load(G.DEFAULT_LUT), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    L = Launch(sched, st.a, st.b, [s.out_dtype for s in st.specs])
+    L.run()
+    got = L.results()
+    rng = np.random.default_rng(j)
+    for i, s in enumerate(st.specs):
+        rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(6, s.M))]))
+        check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} gemm {i} {s.M}x{s.N}x{s.K}")

@@ -1,0 +1,95 @@
+"""The dynamic logic against the paper's "Oracle" configuration (Sec. 5.4:
+always the right concurrency degree, sequential included), made exhaustive.
+
+For small sets the time of every subset run as one concurrent (fused) group,
+each GEMM with the table's GO-Kernel for that group size, is measured on the
+GPU; the oracle's brute-force search (oracle/schedule.py) then finds the best
+split into consecutive groups under those times, and the planner's own
+schedule is timed directly.  The regret (planner / best - 1) must stay small;
+the paper reports its predictor within 3% geomean of its Oracle.  Results are
+also written to gpurun_out/regret.json when that folder exists."""
+import json
+import math
+import os
+
+import pytest
+import torch
+
+import bench
+from oracle import planner_ref as pr
+from oracle import schedule as sch
+from paper_2409_02227_gb300 import goldy as G
+from paper_2409_02227_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+SETS = ["pair_256", "hetero_pair", "sweep_01", "sweep_06", "sweep_15", "sweep_35", "sweep_44"]
+
+
+def _set(name):
+    if name.startswith("sweep_"):
+        return wl.make_sweep_set(int(name.split("_")[1]))
+    return wl.make_config(name)
+
+
+def _time(st, descs, groups, variants, slots, idx, copies=4, steps=60):
+    """Makespan (us) of the sub-set `idx` of `st` under an explicit fused schedule."""
+    sub = wl.GemmSet(st.name, st.seed, [st.specs[i] for i in idx], [st.a[i] for i in idx], [st.b[i] for i in idx])
+    sched = G.goldy_schedule_build([descs[i] for i in idx], groups, variants, slots, G.GOLDY_PLAN_FUSED)
+    r = bench.SetRunner(sub, sched, copies)
+    for k in range(5):
+        r.launch(k)
+    torch.cuda.synchronize()
+    t = r.timed(steps)[0] / steps * 1e3
+    del r
+    return t
+
+
+@pytest.mark.parametrize("name", SETS)
+def test_planner_regret_vs_exhaustive_oracle(cuda_ok, name):
+    st = _set(name)
+    n = len(st.specs)
+    assert n <= 4
+    lut_bytes = open(G.DEFAULT_LUT, "rb").read()
+    entries, _ = pr.parse_lut(lut_bytes)
+    keys = [pr.bucket_key(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+
+    def go_variant(i, size):
+        return pr.lookup(entries, keys[i]).variants[pr.cd_class_index(size)]
+
+    cache = {}
+
+    def group_time(block, variants):
+        if block not in cache:
+            k = len(block)
+            cache[block] = _time(st, descs, [0] * k, list(variants), list(range(k)), list(block))
+        return cache[block]
+
+    best = sch.brute_force(n, lambda i, blk: [go_variant(i, len(blk))], group_time)
+    dp = sch.subset_dp(n, lambda i, blk: [go_variant(i, len(blk))], group_time)
+    assert best.makespan == pytest.approx(dp)
+
+    plan = G.goldy_plan(descs, G.goldy_lut_from_memory(lut_bytes), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    entries_plan = [G.goldy_schedule_entry(plan, i) for i in range(n)]
+    r = bench.SetRunner(st, plan, 4)
+    for k in range(5):
+        r.launch(k)
+    torch.cuda.synchronize()
+    t_plan = r.timed(60)[0] / 60 * 1e3
+    del r
+    # the oracle's schedule, timed the same way (its groups one after another)
+    t_best = 0.0
+    for blk in best.partition:
+        t_best += cache[blk]
+    regret = t_plan / t_best - 1.0
+    record = {"set": name, "n": n, "planner_us": t_plan, "oracle_us": t_best, "regret": regret,
+              "oracle_partition": [list(b) for b in best.partition],
+              "planner_groups": [e[0] for e in entries_plan],
+              "subset_us": {",".join(map(str, k)): v for k, v in cache.items()}}
+    out = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "gpurun_out")
+    if os.path.isdir(out):
+        with open(os.path.join(out, "regret.jsonl"), "a") as f:
+            f.write(json.dumps(record) + "\n")
+    assert math.isfinite(regret)
+    assert regret < 0.35, record
