@@ -331,6 +331,47 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
   }
 }
 
+// Cluster split-K with the partial tiles in shared memory: as reduce_slice,
+// but partial s is read from the shared memory of cluster CTA s (same
+// [chunk][float4][row] layout at `part_smem` in every CTA).
+template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
+__device__ __forceinline__ void reduce_slice_dsmem(const GemmWork& w, uint32_t part_smem, int rank, int m0, int n0,
+                                                   int t) {
+  constexpr int R = 128 / S;
+  constexpr int COLS4 = MMA_N / 4;
+  constexpr int PER_THREAD = R * COLS4 / 128;
+  constexpr int IB = (16 / S < PER_THREAD) ? 16 / S : PER_THREAD;
+  static_assert(PER_THREAD >= 1 && PER_THREAD % IB == 0, "reduce tiling");
+  const int r0 = rank * R;
+  uint32_t peer[S];
+#pragma unroll
+  for (int s2 = 0; s2 < S; ++s2) peer[s2] = ptx::map_to_rank(part_smem, uint32_t(s2));
+#pragma unroll 1
+  for (int k0 = 0; k0 < PER_THREAD; k0 += IB) {
+    float4 vals[IB][S];
+#pragma unroll
+    for (int b = 0; b < IB; ++b) {
+      const int i = t + 128 * (k0 + b);
+      const uint32_t off = uint32_t((i / R) * 128 + r0 + (i % R)) * 16u;
+#pragma unroll
+      for (int s2 = 0; s2 < S; ++s2) vals[b][s2] = ptx::ld_shared_cluster_v4(peer[s2] + off);
+    }
+#pragma unroll
+    for (int b = 0; b < IB; ++b) {
+      const int i = t + 128 * (k0 + b);
+      float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+      for (int s2 = 0; s2 < S; ++s2) {
+        a.x += vals[b][s2].x;
+        a.y += vals[b][s2].y;
+        a.z += vals[b][s2].z;
+        a.w += vals[b][s2].w;
+      }
+      store_quad<SWAP, OUT_BF16>(w, m0, n0, r0 + (i % R), 4 * (i / R), a);
+    }
+  }
+}
+
 template <int MMA_N, int ACC>
 struct TmemCols {
   static constexpr uint32_t need = uint32_t(MMA_N * ACC);
@@ -357,6 +398,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   static_assert(STAGES <= 32, "stage bitmasks");
   static_assert(!(EPI_TMA && SWAP), "the TMA-store epilogue writes untransposed tiles");
   constexpr int STAGING_BYTES = EPI_TMA ? 2 * 16384 : 0;
+  // a whole fp32 partial tile fits in the ring's shared memory
+  constexpr bool kPartFitsRing = STAGES * STAGE_BYTES >= 128 * MMA_N * 4;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -564,6 +607,49 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
           store_chunk<SWAP, OUT_BF16>(w, m0, n0, r, c0, v);
+        }
+      } else if (kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x)) {
+        // ---- cluster split-K on chip: one unit per CTA, so the ring's shared
+        // memory is free once the accumulator is complete.  Publish the fp32
+        // partial there, signal every peer, wait for all S partials, reduce
+        // this CTA's rows reading the peers' shared memory.  The cluster
+        // barrier at kernel exit keeps every CTA resident until its peers are
+        // done reading.
+        const uint32_t part_smem = tiles_base;
+#pragma unroll 1
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int j4 = 0; j4 < 8; ++j4)
+            ptx::st_shared_v4(part_smem + uint32_t(((c0 / 4) + j4) * 128 + r) * 16u, raw[4 * j4],
+                              raw[4 * j4 + 1], raw[4 * j4 + 2], raw[4 * j4 + 3]);
+        }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
+        released = true;
+        ptx::fence_acq_rel_cluster();
+        ptx::named_bar_sync(1, 128);
+        const uint32_t rb = ptx::smem_u32(&redbar[red_it & 1]);
+        if (et == 0) {
+          if (first_unit) trace_stamp(trace, kTrPartials);
+          for (int q2 = 0; q2 < w.split; ++q2) ptx::mbar_arrive_remote_release(ptx::map_to_rank(rb, uint32_t(q2)));
+        }
+        bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag);
+        ok2 = ptx::named_bar_and(1, 128, ok2);
+        ++red_it;
+        if (!ok2) {
+          if (et == 0) raise_error(p.err, abort_flag, kErrClusterWait);
+          break;
+        }
+        if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
+        switch (w.split) {
+          case 2: reduce_slice_dsmem<MMA_N, 2, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
+          case 4: reduce_slice_dsmem<MMA_N, 4, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
+          case 8: reduce_slice_dsmem<MMA_N, 8, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
+          default: break;
         }
       } else {
         // partial tile layout: [chunk][float4 index j4][row r] -> coalesced per warp
