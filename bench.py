@@ -3,7 +3,9 @@
 
 One step = one pass of the whole hot path over one synthetic GEMM set: the
 dynamic logic's plan (computed once; it is a pure function of the shapes)
-replayed as a CUDA graph of GO-Kernel launches on CD streams.  Default
+replayed as a prepared run of GO-Kernel launches on CD streams (recorded
+once, replayed with plain launches; ``--replay graph`` replays a captured
+CUDA graph instead).  Default
 workload: the tensor-sliced Transformer FFN at low batch, 4 independent
 GEMMs of M=128, N=1024, K=4096, bf16 in, fp32 accumulate, bf16 out.
 
@@ -54,6 +56,8 @@ def parse_args(argv=None):
     ap.add_argument("--lut", default=None, help="lookup table (default: the packaged one)")
     ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
                     help="fused: a wave's same-kind GEMMs share one launch; streams: one launch per GEMM")
+    ap.add_argument("--replay", choices=["exec", "graph"], default="exec",
+                    help="how the prepared step is replayed: recorded plain launches or a CUDA graph")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--report", default=None, metavar="FILE",
@@ -269,14 +273,17 @@ def run_reference(args, world, rank):
 
 # ----------------------------------------------------------------------------- GPU arm
 class SetRunner:
-    """R rotating device copies of one GEMM set, one captured graph per copy."""
+    """R rotating device copies of one GEMM set, each with its run prepared
+    once: a recorded prepared run (``replay="exec"``, plain launches) or a
+    captured CUDA graph (``replay="graph"``)."""
 
-    def __init__(self, st, sched, copies, with_events=False):
+    def __init__(self, st, sched, copies, with_events=False, replay="exec"):
         import torch
         from paper_2409_02227_gb300 import goldy as G
         self.G = G
         self.torch = torch
         self.sched = sched
+        self.replay = replay
         n, _, ms, ws_bytes = G.goldy_schedule_query(sched)
         self.n = n
         self.ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
@@ -292,32 +299,40 @@ class SetRunner:
             C = [torch.empty((s.M, s.N), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
             self.copies.append((A, B, C))
         self.events = []
-        self.graphs = []
+        self.runs = []
         torch.cuda.synchronize()
+        sp = [s.cuda_stream for s in self.streams]
         for A, B, C in self.copies:
             ptrs = ([a.data_ptr() for a in A], [b.data_ptr() for b in B], [c.data_ptr() for c in C])
+            evs = {}
             if with_events:
                 eb = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
                 ee = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
                 for e in eb + ee:            # torch creates the CUDA event on first record
                     e.record()
                 torch.cuda.synchronize()
-                g = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes,
-                                            [s.cuda_stream for s in self.streams],
-                                            [e.cuda_event for e in eb], [e.cuda_event for e in ee])
+                evs = {"ev_begin": [e.cuda_event for e in eb], "ev_end": [e.cuda_event for e in ee]}
                 self.events.append((eb, ee))
+            if replay == "exec":
+                r = G.goldy_exec_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp, **evs)
+            elif evs:
+                r = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp,
+                                            evs["ev_begin"], evs["ev_end"])
             else:
-                g = G.goldy_graph_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes,
-                                         [s.cuda_stream for s in self.streams])
-            self.graphs.append(g)
+                r = G.goldy_graph_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp)
+            self.runs.append(r)
         self.main = self.streams[0]
 
     def __del__(self):
-        # destroy the graphs before the buffers they read and write
-        self.graphs.clear()
+        # destroy the prepared runs before the buffers they read and write
+        self.runs.clear()
 
     def launch(self, k):
-        self.G.goldy_graph_launch(self.graphs[k % len(self.graphs)], self.main.cuda_stream)
+        r = self.runs[k % len(self.runs)]
+        if self.replay == "exec":
+            self.G.goldy_exec_launch(r)
+        else:
+            self.G.goldy_graph_launch(r, self.main.cuda_stream)
 
     def timed(self, steps, step_events=0):
         """Elapsed ms of `steps` back-to-back replays; with `step_events`, the
@@ -453,7 +468,7 @@ def run_gpu(args, world, rank, local):
     in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
     copies = max(2, math.ceil(2 * l2 / in_bytes))
 
-    runner = SetRunner(st, sched, copies)
+    runner = SetRunner(st, sched, copies, replay=args.replay)
     for k in range(max(3, args.warmup)):
         runner.launch(k)
     torch.cuda.synchronize()
@@ -485,19 +500,22 @@ def run_gpu(args, world, rank, local):
     dom_v = max(by_variant, key=lambda v: sum(st.specs[i].flops for i in by_variant[v]))
     dom_idx = by_variant[dom_v]
     if single_launch:
-        # one launch per step: the events around each of the last 64 timed
-        # replays on the launching stream time that launch; it covers all GEMMs
-        durs = step_ms
+        # one launch per step, covering all GEMMs: its average duration is the
+        # timed region's elapsed time over the steps (gaps between launches
+        # included, so an upper bound); events around each of the last 64
+        # steps are reported beside it (they add a gap of their own)
+        durs = [ms_step]
         dom_idx = list(range(len(descs)))
-        timing_note = "events around the single fused launch of each of the last 64 timed steps"
+        timing_note = (f"timed-region events / steps (one launch per step); events around each of the last "
+                       f"{len(step_ms)} steps alone: {statistics.mean(step_ms) * 1e3:.2f} us")
     else:
-        inst = SetRunner(st, sched, copies, with_events=True)
+        inst = SetRunner(st, sched, copies, with_events=True, replay=args.replay)
         for k in range(2 * copies):
             inst.launch(k)
         torch.cuda.synchronize()
         durs = [eb[i].elapsed_time(ee[i]) for eb, ee in inst.events for i in dom_idx]
         del inst
-        timing_note = "events recorded around each launch on its own stream inside an instrumented copy of the graph"
+        timing_note = "events recorded around each launch on its own stream inside an instrumented copy of the run"
     dur_ms = statistics.mean(durs)
     bytes_per_launch = sum(st.specs[i].bytes for i in dom_idx) / (1 if single_launch else len(dom_idx))
     flops_per_launch = sum(st.specs[i].flops for i in dom_idx) / (1 if single_launch else len(dom_idx))
@@ -513,7 +531,8 @@ def run_gpu(args, world, rank, local):
         roof = {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
                 "frac": achieved / tf_burst}
     roof["traffic"] = recorded_traffic(vname)
-    roof.update({"kernel": vname, "launch_us": dur_ms * 1e3, "launches_sampled": len(durs),
+    roof.update({"kernel": vname, "launch_us": dur_ms * 1e3,
+                 "launches_sampled": args.steps if single_launch else len(durs),
                  "timing": timing_note,
                  "per_launch": {"algorithmic_bytes": bytes_per_launch, "flops": flops_per_launch},
                  "peak_source": f"{peak_src} ({'HBM copy' if roof['bound'] == 'hbm' else 'cuBLAS bf16 burst'})"})
@@ -527,7 +546,8 @@ def run_gpu(args, world, rank, local):
         "config": {"workload": f"{args.config}: {workload_label(st.specs)}",
                    "l2": f"inputs larger than L2: {copies} rotating device copies of the set "
                          f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2)",
-                   "launch": f"CUDA graph replay of the planned schedule ({args.launch} launch mode)",
+                   "launch": f"{'prepared-run' if args.replay == 'exec' else 'CUDA graph'} replay of the planned "
+                             f"schedule ({args.launch} launch mode)",
                    "plan": [{"gemm": i, "group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl,
                              "cd": cd} for i, (g, v, sl, cd) in enumerate(plan)],
                    "parallelism": f"replicas x{world}"},
@@ -548,12 +568,19 @@ def run_gpu(args, world, rank, local):
                             ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
                             ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
             s2 = G.goldy_plan(descs, lut, flags)
-            r2 = SetRunner(st, s2, copies)
+            r2 = SetRunner(st, s2, copies, replay=args.replay)
             for k in range(10):
                 r2.launch(k)
             torch.cuda.synchronize()
             comp[name] = r2.timed(csteps)[0] / csteps * 1e3
             del r2
+        other = "graph" if args.replay == "exec" else "exec"
+        r2 = SetRunner(st, sched, copies, replay=other)
+        for k in range(10):
+            r2.launch(k)
+        torch.cuda.synchronize()
+        comp[f"planned_schedule_{other}_replay"] = r2.timed(csteps)[0] / csteps * 1e3
+        del r2
         a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
         cb = cublas_reference_ms(st, copies, csteps) * 1e3
         line["comparisons_us"] = {**comp, "cublas_sequential_reference": cb}
@@ -579,7 +606,7 @@ def run_gpu(args, world, rank, local):
     return 0
 
 
-def time_policies(st, lut, copies, steps):
+def time_policies(st, lut, copies, steps, replay="exec"):
     """Makespan (us) of one set under each policy, timed like the main line."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
@@ -591,7 +618,7 @@ def time_policies(st, lut, copies, steps):
                         ("naive_streams", G.GOLDY_PLAN_DEFAULT),
                         ("go_all_concurrent", G.GOLDY_PLAN_GO)):
         sched = G.goldy_plan(descs, lut, flags)
-        r = SetRunner(st, sched, copies)
+        r = SetRunner(st, sched, copies, replay=replay)
         for k in range(10):
             r.launch(k)
         torch.cuda.synchronize()
@@ -622,7 +649,7 @@ def run_report(args, local):
         in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
         copies = max(2, math.ceil(2 * l2 / in_bytes))
         steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
-        t = time_policies(st, lut, copies, steps)
+        t = time_policies(st, lut, copies, steps, args.replay)
         if name in wl.FIXED_CONFIGS:
             t["cublas_sequential_reference"] = cublas_reference_ms(st, copies, steps) * 1e3
         roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6

@@ -233,6 +233,22 @@ goldy_status goldy_run_ex(const goldy_schedule* s, const void* const* A, const v
                           void* const* C, void* workspace, size_t workspace_bytes,
                           void* const* streams, int n_streams, const goldy_run_opts* opts);
 
+/* Prepared run: record goldy_run_ex(...) with these exact pointers and
+ * streams once — tensor maps encoded, kernel parameter blocks built, grids and
+ * cluster shapes fixed, fork/join events owned by the object — so that
+ * goldy_exec_launch replays it with plain launch calls on the same streams.
+ * On this platform a replay costs about half of a one-kernel CUDA graph
+ * launch.  Nothing is launched by goldy_exec_create; the buffers and streams
+ * must outlive the object.  Not thread-safe per object. */
+typedef struct goldy_exec goldy_exec;
+goldy_status goldy_exec_create(const goldy_schedule* s, const void* const* A, const void* const* B,
+                               void* const* C, void* workspace, size_t workspace_bytes,
+                               void* const* streams, int n_streams, const goldy_run_opts* opts,
+                               goldy_exec** out);
+/* Enqueue a prepared run (asynchronous, no allocation). */
+goldy_status goldy_exec_launch(const goldy_exec* e);
+void goldy_exec_free(goldy_exec* e);
+
 /* Capture goldy_run(...) with these exact pointers into a CUDA graph, for
  * replay with one launch (the closest host-side analogue of the command
  * processor dispatching a whole set).  The streams must be idle.  The graph

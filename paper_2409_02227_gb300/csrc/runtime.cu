@@ -21,7 +21,9 @@
 #include <algorithm>
 #include <cstring>
 #include <mutex>
+#include <new>
 #include <string>
+#include <vector>
 
 #include "go_kernel.cuh"
 #include "goldy_internal.h"
@@ -42,6 +44,26 @@ void runtime_release(Runtime* rt) {
   for (cudaEvent_t e : rt->join)
     if (e) cudaEventDestroy(e);
   delete rt;
+}
+
+// One enqueued operation of a run.  goldy_run_ex executes them as it goes;
+// goldy_exec_create records them (with copies of the kernel parameter blocks)
+// so goldy_exec_launch can replay the run with plain launch calls.
+struct Op {
+  enum Kind { kKernel, kMemset2D, kEventRecord, kEventRecordExternal, kWait } kind = kKernel;
+  cudaStream_t stream = nullptr;
+  const void* fn = nullptr;
+  unsigned grid = 0;
+  size_t smem = 0;
+  int cluster = 0;
+  std::vector<uint64_t> params;      // 8-byte-aligned copy of the parameter block
+  void* ptr = nullptr;
+  size_t pitch = 0, width = 0, height = 0;
+  cudaEvent_t ev = nullptr;
+};
+
+namespace {
+thread_local std::vector<Op>* t_rec = nullptr;   // non-null: record instead of enqueue
 }
 
 namespace {
@@ -134,7 +156,8 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
 
 // Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
 // cluster > 1.
-cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params, int cluster) {
+cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params,
+                              int cluster) {
   void* args[] = {params};
   if (cluster <= 1) return cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream);
   cudaLaunchConfig_t cfg = {};
@@ -150,6 +173,74 @@ cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
+cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, const void* params,
+                          size_t params_size, int cluster) {
+  if (!t_rec) return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster);
+  Op op;
+  op.kind = Op::kKernel;
+  op.stream = stream;
+  op.fn = fn;
+  op.grid = grid;
+  op.smem = smem;
+  op.cluster = cluster;
+  op.params.resize((params_size + 7) / 8);
+  std::memcpy(op.params.data(), params, params_size);
+  t_rec->push_back(std::move(op));
+  return cudaSuccess;
+}
+
+cudaError_t enq_memset2d(void* ptr, size_t pitch, size_t width, size_t height, cudaStream_t stream) {
+  if (!t_rec) return cudaMemset2DAsync(ptr, pitch, 0, width, height, stream);
+  Op op;
+  op.kind = Op::kMemset2D;
+  op.stream = stream;
+  op.ptr = ptr;
+  op.pitch = pitch;
+  op.width = width;
+  op.height = height;
+  t_rec->push_back(std::move(op));
+  return cudaSuccess;
+}
+
+cudaError_t enq_event_record(cudaEvent_t ev, cudaStream_t stream, bool external = false) {
+  if (!t_rec) {
+    if (!external) return cudaEventRecord(ev, stream);
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(stream, &cs);
+    if (e != cudaSuccess) return e;
+    return cudaEventRecordWithFlags(ev, stream, cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : 0);
+  }
+  Op op;
+  op.kind = external ? Op::kEventRecordExternal : Op::kEventRecord;
+  op.stream = stream;
+  op.ev = ev;
+  t_rec->push_back(std::move(op));
+  return cudaSuccess;
+}
+
+cudaError_t enq_wait(cudaStream_t stream, cudaEvent_t ev) {
+  if (!t_rec) return cudaStreamWaitEvent(stream, ev, 0);
+  Op op;
+  op.kind = Op::kWait;
+  op.stream = stream;
+  op.ev = ev;
+  t_rec->push_back(std::move(op));
+  return cudaSuccess;
+}
+
+cudaError_t replay(const Op& op) {
+  switch (op.kind) {
+    case Op::kKernel:
+      return launch_kernel_now(op.fn, op.grid, op.smem, op.stream, const_cast<uint64_t*>(op.params.data()),
+                               op.cluster);
+    case Op::kMemset2D: return cudaMemset2DAsync(op.ptr, op.pitch, 0, op.width, op.height, op.stream);
+    case Op::kEventRecord: return cudaEventRecord(op.ev, op.stream);
+    case Op::kEventRecordExternal: return cudaEventRecordWithFlags(op.ev, op.stream, 0);
+    case Op::kWait: return cudaStreamWaitEvent(op.stream, op.ev, 0);
+  }
+  return cudaErrorInvalidValue;
 }
 
 // Can clusters of `cluster` CTAs of this kernel be resident at all?
@@ -253,7 +344,7 @@ goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream)
   const goldy_gemm_desc& g = gp.desc;
   if (g.M == 0 || g.N == 0) return GOLDY_OK;
   const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
-  cudaError_t e = cudaMemset2DAsync(C, size_t(g.ldc) * es, 0, size_t(g.N) * es, size_t(g.M), stream);
+  cudaError_t e = enq_memset2d(C, size_t(g.ldc) * es, size_t(g.N) * es, size_t(g.M), stream);
   return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
 }
 
@@ -291,7 +382,8 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   if (k.pair) {
     const unsigned grid = pair_grid(gp.units, cap);
     p.trace = trace_for(grid);
-    cudaError_t e = launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, 2);
+    cudaError_t e =
+        launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, sizeof(p), 2);
     if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (pair)");
     return GOLDY_OK;
   }
@@ -299,7 +391,8 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   p.cluster = cluster;
   const unsigned grid = launch_grid(gp.units, cap, cluster);
   p.trace = trace_for(grid);
-  cudaError_t e = launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, cluster);
+  cudaError_t e =
+      launch_kernel(kernel_fn(gp.kind, out_bf16, 0), grid, size_t(smem_bytes(k)), stream, &p, sizeof(p), cluster);
   if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel");
   return GOLDY_OK;
 }
@@ -336,7 +429,8 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   if (k.pair) {
     const unsigned grid = pair_grid(units, cap);
     p.trace = trace_for(grid);
-    cudaError_t e = launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, 2);
+    cudaError_t e =
+        launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, sizeof(p), 2);
     if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (fused pair)");
     return GOLDY_OK;
   }
@@ -348,7 +442,8 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.cluster = cluster;
   const unsigned grid = launch_grid(units, cap, cluster);
   p.trace = trace_for(grid);
-  cudaError_t e = launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, cluster);
+  cudaError_t e =
+      launch_kernel(kernel_fn(g0.kind, out_bf16, 1), grid, size_t(smem_bytes(k)), stream, &p, sizeof(p), cluster);
   if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (fused)");
   return GOLDY_OK;
 }
@@ -363,11 +458,7 @@ namespace {
 // external record to become a real node of the graph.
 cudaError_t record_hook(void* ev, cudaStream_t stream) {
   if (!ev) return cudaSuccess;
-  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  cudaError_t e = cudaStreamIsCapturing(stream, &cs);
-  if (e != cudaSuccess) return e;
-  return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev), stream,
-                                  cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : 0);
+  return enq_event_record(static_cast<cudaEvent_t>(ev), stream, true);
 }
 }  // namespace
 
@@ -377,9 +468,28 @@ extern "C" goldy_status goldy_run(const goldy_schedule* s, const void* const* A,
   return goldy_run_ex(s, A, B, C, workspace, workspace_bytes, streams, n_streams, nullptr);
 }
 
-extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const* A, const void* const* B,
-                                     void* const* C, void* workspace, size_t workspace_bytes, void* const* streams,
-                                     int n_streams, const goldy_run_opts* opts) {
+namespace goldy {
+Runtime* new_runtime(int dev, goldy_status* st) {
+  Runtime* rt = new Runtime();
+  rt->device = dev;
+  cudaError_t e = cudaEventCreateWithFlags(&rt->fork, cudaEventDisableTiming);
+  for (int k = 0; k < GOLDY_MAX_STREAMS && e == cudaSuccess; ++k)
+    e = cudaEventCreateWithFlags(&rt->join[k], cudaEventDisableTiming);
+  if (e != cudaSuccess) {
+    runtime_release(rt);
+    *st = cuda_fail(e, "cudaEventCreate");
+    return nullptr;
+  }
+  *st = GOLDY_OK;
+  return rt;
+}
+}  // namespace goldy
+
+// The run itself; `own_rt`, if given, supplies the fork/join events (a
+// recorded run owns its events), otherwise the schedule's are used.
+static goldy_status run_impl(const goldy_schedule* s, const void* const* A, const void* const* B, void* const* C,
+                             void* workspace, size_t workspace_bytes, void* const* streams, int n_streams,
+                             const goldy_run_opts* opts, Runtime* own_rt) {
   if (!s || !A || !B || !C || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
   if (n_streams < s->max_streams) return fail(GOLDY_ERR_INVALID_ARG, "fewer streams than the schedule needs");
   if (s->workspace_bytes > 0) {
@@ -400,26 +510,21 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
   goldy_status st = device_state(&d);
   if (st != GOLDY_OK) return st;
 
-  goldy_schedule* ms = const_cast<goldy_schedule*>(s);
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (ms->rt && ms->rt->device != dev) {
-    runtime_release(ms->rt);
-    ms->rt = nullptr;
-  }
-  if (!ms->rt) {
-    Runtime* rt = new Runtime();
-    rt->device = dev;
-    cudaError_t e = cudaEventCreateWithFlags(&rt->fork, cudaEventDisableTiming);
-    for (int k = 0; k < GOLDY_MAX_STREAMS && e == cudaSuccess; ++k)
-      e = cudaEventCreateWithFlags(&rt->join[k], cudaEventDisableTiming);
-    if (e != cudaSuccess) {
-      runtime_release(rt);
-      return cuda_fail(e, "cudaEventCreate");
+  Runtime* rt = own_rt;
+  if (!rt) {
+    goldy_schedule* ms = const_cast<goldy_schedule*>(s);
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (ms->rt && ms->rt->device != dev) {
+      runtime_release(ms->rt);
+      ms->rt = nullptr;
     }
-    ms->rt = rt;
+    if (!ms->rt) {
+      ms->rt = new_runtime(dev, &st);
+      if (!ms->rt) return st;
+    }
+    rt = ms->rt;
   }
-  Runtime* rt = ms->rt;
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
 
@@ -499,11 +604,11 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
     for (int t = 0; t < n_sets; ++t) used |= 1u << sets[t].slot;
     const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
     if (side) {
-      cudaError_t e = cudaEventRecord(rt->fork, main);
+      cudaError_t e = enq_event_record(rt->fork, main);
       if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
       for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
         if (side >> k & 1) {
-          e = cudaStreamWaitEvent(static_cast<cudaStream_t>(streams[k]), rt->fork, 0);
+          e = enq_wait(static_cast<cudaStream_t>(streams[k]), rt->fork);
           if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
         }
     }
@@ -525,8 +630,8 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
     if (side) {
       for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
         if (side >> k & 1) {
-          cudaError_t e = cudaEventRecord(rt->join[k], static_cast<cudaStream_t>(streams[k]));
-          if (e == cudaSuccess) e = cudaStreamWaitEvent(main, rt->join[k], 0);
+          cudaError_t e = enq_event_record(rt->join[k], static_cast<cudaStream_t>(streams[k]));
+          if (e == cudaSuccess) e = enq_wait(main, rt->join[k]);
           if (e != cudaSuccess) return cuda_fail(e, "join event");
         }
     }
@@ -534,6 +639,62 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
   t_trace = nullptr;
   t_trace_ctas = 0;
   return ok();
+}
+
+extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                     void* const* C, void* workspace, size_t workspace_bytes, void* const* streams,
+                                     int n_streams, const goldy_run_opts* opts) {
+  return run_impl(s, A, B, C, workspace, workspace_bytes, streams, n_streams, opts, nullptr);
+}
+
+struct goldy_exec {
+  std::vector<Op> ops;
+  Runtime* rt = nullptr;
+};
+
+extern "C" goldy_status goldy_exec_create(const goldy_schedule* s, const void* const* A, const void* const* B,
+                                          void* const* C, void* workspace, size_t workspace_bytes,
+                                          void* const* streams, int n_streams, const goldy_run_opts* opts,
+                                          goldy_exec** out) {
+  if (!out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  goldy_status st = GOLDY_OK;
+  goldy_exec* x = new (std::nothrow) goldy_exec();
+  if (!x) return fail(GOLDY_ERR_NOMEM, "out of host memory");
+  x->rt = new_runtime(dev, &st);
+  if (!x->rt) {
+    delete x;
+    return st;
+  }
+  t_rec = &x->ops;
+  st = run_impl(s, A, B, C, workspace, workspace_bytes, streams, n_streams, opts, x->rt);
+  t_rec = nullptr;
+  if (st != GOLDY_OK) {
+    std::string why = goldy_last_error();
+    runtime_release(x->rt);
+    delete x;
+    return fail(st, why);
+  }
+  *out = x;
+  return ok();
+}
+
+extern "C" goldy_status goldy_exec_launch(const goldy_exec* x) {
+  if (!x) return fail(GOLDY_ERR_INVALID_ARG, "null exec");
+  for (const Op& op : x->ops) {
+    cudaError_t e = replay(op);
+    if (e != cudaSuccess) return cuda_fail(e, "goldy_exec_launch");
+  }
+  return ok();
+}
+
+extern "C" void goldy_exec_free(goldy_exec* x) {
+  if (!x) return;
+  runtime_release(x->rt);
+  delete x;
 }
 
 struct goldy_graph {

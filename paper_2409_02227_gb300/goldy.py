@@ -102,6 +102,9 @@ def _load():
         "goldy_run_ex": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts)], I),
         "goldy_graph_create_ex": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts), PP], I),
         "goldy_graph_launch": ([P, P], I),
+        "goldy_exec_create": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts), PP], I),
+        "goldy_exec_launch": ([P], I),
+        "goldy_exec_free": ([P], None),
         "goldy_graph_free": ([P], None),
         "goldy_gemm_noalloc": ([DP, I, P, P, P, P], I),
         "goldy_device_error": ([IP, I], I),
@@ -171,6 +174,10 @@ class Schedule(_Handle):
 
 class Graph(_Handle):
     _free = staticmethod(lambda p: _lib.goldy_graph_free(p))
+
+
+class Exec(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_exec_free(p))
 
 
 def goldy_abi_version() -> int:
@@ -305,6 +312,21 @@ def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Se
                                       int(workspace_bytes), _ptrs(streams), len(streams),
                                       ctypes.byref(o), ctypes.byref(out)), "goldy_graph_create_ex")
     return Graph(out)
+
+
+def goldy_exec_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
+                      workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
+                      ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0) -> Exec:
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas)
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_exec_create(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
+                                  int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o),
+                                  ctypes.byref(out)), "goldy_exec_create")
+    return Exec(out)
+
+
+def goldy_exec_launch(e: Exec) -> None:
+    _check(_lib.goldy_exec_launch(e.ptr), "goldy_exec_launch")
 
 
 def goldy_graph_launch(g: Graph, stream: int) -> None:

@@ -43,6 +43,11 @@ class Launch:
         return G.goldy_graph_create(self.sched, A, B, C, self.ws.data_ptr(), self.ws_bytes,
                                     [s.cuda_stream for s in self.streams])
 
+    def exec(self):
+        A, B, C = self.ptrs()
+        return G.goldy_exec_create(self.sched, A, B, C, self.ws.data_ptr(), self.ws_bytes,
+                                   [s.cuda_stream for s in self.streams])
+
     def results(self):
         torch.cuda.synchronize()
         err = G.goldy_device_error(clear=True)

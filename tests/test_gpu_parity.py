@@ -135,6 +135,34 @@ def test_graph_replay_matches_eager(cuda_ok):
         assert torch.equal(e.view(torch.int16), x.view(torch.int16))
 
 
+@pytest.mark.parametrize("fused", [False, True])
+def test_exec_replay_matches_eager(cuda_ok, fused):
+    """A prepared run (recorded once, replayed with plain launches) gives the
+    eager run's bits, over several replays, on split-K, cluster and pair
+    variants with a degenerate member in the set."""
+    shapes = [(128, 1024, 4096), (256, 512, 2048), (100, 384, 1000), (0, 128, 64)]
+    A, B = zip(*[inputs(M, N, K, seed=650 + i, dist="normal", scale=0.02) for i, (M, N, K) in enumerate(shapes)])
+    vs = [vid(1, 4, 4), vid(10, 1, 4), vid(3, 2, 4), vid(2)]
+    descs = [G.desc(M, N, K, BF16) for (M, N, K) in shapes]
+    s = G.goldy_schedule_build(descs, [0] * 4, vs, [0, 1, 2, 3], G.GOLDY_PLAN_FUSED if fused else 0)
+    L = Launch(s, list(A), list(B), [BF16] * 4)
+    L.run()
+    eager = [c.clone() for c in L.results()]
+    L.streams[0].wait_stream(torch.cuda.current_stream())
+    x = L.exec()
+    for c in L.dC:
+        c.fill_(float("nan"))
+    L.streams[0].wait_stream(torch.cuda.current_stream())
+    for _ in range(3):
+        G.goldy_exec_launch(x)
+    torch.cuda.current_stream().wait_stream(L.streams[0])
+    got = L.results()
+    for e, g in zip(eager, got):
+        assert torch.equal(e.view(torch.int16), g.view(torch.int16))
+    check_close(got[1].float(), A[1], B[1], "exec pair")
+    del x
+
+
 def test_degenerate_sizes(cuda_ok):
     a0 = torch.zeros((0, 64), dtype=torch.bfloat16)
     b0 = wl.random_matrix(64, 128, seed=1)
