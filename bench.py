@@ -60,6 +60,8 @@ def parse_args(argv=None):
                     help="how the prepared step is replayed: recorded plain launches or a CUDA graph")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--scaling-study", default=None, metavar="FILE",
+                    help="GPU-scaling study inside SM partitions of 1/4, 1/2 and all of the GPU (JSON to FILE)")
     ap.add_argument("--report", default=None, metavar="FILE",
                     help="instead of the JSON line: time every fixed set and the 64 randomized sets "
                          "under every policy and write a JSON report to FILE (markdown table on stdout)")
@@ -364,6 +366,23 @@ class SetRunner:
         return out
 
 
+def time_schedule(st, sched, copies, steps, warm=10):
+    """Makespan (us) of one schedule, replayed both ways (recorded plain
+    launches and a CUDA graph); each configuration is credited with its
+    faster replay, so that no baseline is slowed by a launch mode that does
+    not suit it.  Returns (best, {"exec": us, "graph": us})."""
+    import torch
+    out = {}
+    for mode in ("exec", "graph"):
+        r = SetRunner(st, sched, copies, replay=mode)
+        for k in range(warm):
+            r.launch(k)
+        torch.cuda.synchronize()
+        out[mode] = r.timed(steps)[0] / steps * 1e3
+        del r
+    return min(out.values()), out
+
+
 def cublas_reference_ms(st, copies, steps):
     """torch.matmul (cuBLAS) for the same set, back to back on one stream,
     captured in a CUDA graph per rotating copy: a reference point only."""
@@ -562,28 +581,18 @@ def run_gpu(args, world, rank, local):
 
     if not args.no_compare:
         csteps = max(200, min(args.steps, 5000))
-        comp = {}
+        comp, modes = {}, {}
         for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
                             ("go_all_concurrent", G.GOLDY_PLAN_GO),
                             ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
                             ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
             s2 = G.goldy_plan(descs, lut, flags)
-            r2 = SetRunner(st, s2, copies, replay=args.replay)
-            for k in range(10):
-                r2.launch(k)
-            torch.cuda.synchronize()
-            comp[name] = r2.timed(csteps)[0] / csteps * 1e3
-            del r2
-        other = "graph" if args.replay == "exec" else "exec"
-        r2 = SetRunner(st, sched, copies, replay=other)
-        for k in range(10):
-            r2.launch(k)
-        torch.cuda.synchronize()
-        comp[f"planned_schedule_{other}_replay"] = r2.timed(csteps)[0] / csteps * 1e3
-        del r2
+            comp[name], modes[name] = time_schedule(st, s2, copies, csteps)
         a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
         cb = cublas_reference_ms(st, copies, csteps) * 1e3
-        line["comparisons_us"] = {**comp, "cublas_sequential_reference": cb}
+        line["comparisons_us"] = {**comp, "cublas_sequential_reference": cb,
+                                  "by_replay": modes,
+                                  "note": "each configuration at its faster replay (recorded launches or graph)"}
         line["speedup_vs_sequential"] = comp["sequential"] / a_us
         line["speedup_vs_naive_streams"] = comp["naive_streams"] / a_us
 
@@ -606,26 +615,29 @@ def run_gpu(args, world, rank, local):
     return 0
 
 
-def time_policies(st, lut, copies, steps, replay="exec"):
+def time_policies(st, lut, copies, steps):
     """Makespan (us) of one set under each policy, timed like the main line."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
     descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
     out = {}
+    predictor = G.goldy_predictor_load() if os.path.exists(G.DEFAULT_PREDICTOR) else None
     for name, flags in (("goldyloc", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED),
+                        ("goldyloc_lr", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED),
                         ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
                         ("sequential", G.GOLDY_PLAN_SEQUENTIAL),
                         ("naive_streams", G.GOLDY_PLAN_DEFAULT),
                         ("go_all_concurrent", G.GOLDY_PLAN_GO)):
-        sched = G.goldy_plan(descs, lut, flags)
-        r = SetRunner(st, sched, copies, replay=replay)
-        for k in range(10):
-            r.launch(k)
-        torch.cuda.synchronize()
-        out[name] = r.timed(steps)[0] / steps * 1e3
-        if name == "goldyloc":
-            out["plan"] = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
-        del r
+        if name == "goldyloc_lr":
+            if predictor is None:
+                continue
+            sched = G.goldy_plan_ex(descs, lut, predictor, flags)
+        else:
+            sched = G.goldy_plan(descs, lut, flags)
+        out[name], out.setdefault("by_replay", {})[name] = time_schedule(st, sched, copies, steps)
+        if name in ("goldyloc", "goldyloc_lr"):
+            out["plan" if name == "goldyloc" else "plan_lr"] = [G.goldy_schedule_entry(sched, i)
+                                                                 for i in range(len(descs))]
     if G.goldy_device_error(clear=True) != 0:
         raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
     return out
@@ -649,27 +661,31 @@ def run_report(args, local):
         in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
         copies = max(2, math.ceil(2 * l2 / in_bytes))
         steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
-        t = time_policies(st, lut, copies, steps, args.replay)
+        t = time_policies(st, lut, copies, steps)
         if name in wl.FIXED_CONFIGS:
             t["cublas_sequential_reference"] = cublas_reference_ms(st, copies, steps) * 1e3
         roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
         row = {"set": name, "n_gemms": len(st.specs), "flops": st.flops, "bytes": st.bytes,
                "bound": "tensor" if st.flops / st.bytes > tf_burst * 1e12 / (hbm * 1e9) else "hbm",
-               "roof_us": roof_us, "us": {k: v for k, v in t.items() if k != "plan"},
+               "roof_us": roof_us,
+               "us": {k: v for k, v in t.items() if not k.startswith("plan") and k != "by_replay"},
+               "us_by_replay": t["by_replay"],
                "tflops": st.flops / (t["goldyloc"] * 1e-6) / 1e12,
                "roofline_frac": roof_us / t["goldyloc"],
                "speedup_vs_sequential": t["sequential"] / t["goldyloc"],
                "speedup_vs_naive_streams": t["naive_streams"] / t["goldyloc"],
                "plan": [{"group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl, "cd": cd}
-                        for g, v, sl, cd in t["plan"]]}
+                        for g, v, sl, cd in t["plan"]],
+               "plan_lr_differs": t.get("plan_lr", t["plan"]) != t["plan"]}
         rows.append(row)
         print(f"| {name} | {len(st.specs)} | {row['bound']} | {roof_us:.2f} | {t['goldyloc']:.2f} | "
               f"{row['tflops']:.1f} | {row['roofline_frac']:.3f} | {row['speedup_vs_sequential']:.2f} | "
-              f"{row['speedup_vs_naive_streams']:.2f} |", flush=True)
+              f"{row['speedup_vs_naive_streams']:.2f} | {t.get('goldyloc_lr', float('nan')):.2f} |", flush=True)
         del st
         torch.cuda.empty_cache()
     sweep = [r for r in rows if r["set"].startswith("sweep")]
     geo = lambda xs: math.exp(sum(math.log(x) for x in xs) / len(xs))
+    lr_rows = [r for r in sweep if "goldyloc_lr" in r["us"]]
     summary = {"sweep_geomean_speedup_vs_sequential": geo([r["speedup_vs_sequential"] for r in sweep]),
                "sweep_geomean_speedup_vs_naive_streams": geo([r["speedup_vs_naive_streams"] for r in sweep]),
                "sweep_geomean_roofline_frac": geo([r["roofline_frac"] for r in sweep]),
@@ -677,9 +693,102 @@ def run_report(args, local):
                                                                 if r["bound"] == "tensor"] or [1.0]),
                "sweep_sets_faster_than_sequential": sum(r["speedup_vs_sequential"] > 1 for r in sweep),
                "sweep_sets_faster_than_naive_streams": sum(r["speedup_vs_naive_streams"] > 1 for r in sweep)}
+    if lr_rows:
+        # the predictor-planned schedule against the table-planned one (Sec. 4.3)
+        summary["sweep_geomean_lr_over_table_time"] = geo([r["us"]["goldyloc_lr"] / r["us"]["goldyloc"]
+                                                           for r in lr_rows])
+        summary["sweep_geomean_lr_speedup_vs_sequential"] = geo([r["us"]["sequential"] / r["us"]["goldyloc_lr"]
+                                                                 for r in lr_rows])
+        summary["sweep_sets_lr_plan_differs"] = sum(r.get("plan_lr_differs", False) for r in lr_rows)
     print(json.dumps(summary), flush=True)
     with open(args.report, "w") as f:
         json.dump({"rows": rows, "summary": summary, "peaks": {"hbm_gbs": hbm, "bf16_tflops": tf_burst}}, f, indent=1)
+    return 0
+
+
+SCALING_PARTITIONS = ((38, "GPU-Quarter"), (76, "GPU-Half"), (0, "GPU"))
+
+
+def scaling_lut_path(sm_count: int) -> str:
+    from paper_2409_02227_gb300 import goldy as G
+    return os.path.join(os.path.dirname(G.DEFAULT_LUT), "scaling", f"goldy_lut_sm{sm_count}.bin")
+
+
+def run_scaling_study(args, local):
+    """GPU-scaling study (Sec. 6.7): each study set (4 equal GEMMs, CD 4) run
+    inside SM partitions of a quarter, half and all of the GPU, under the
+    default configuration (isolation-tuned kernels, all GEMMs on their own
+    streams), sequential, GOLDYLOC with the table tuned inside that partition,
+    and GOLDYLOC re-using the whole-GPU table.  Everything is timed inside the
+    partition (prepared runs, events in the partition)."""
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2409_02227_gb300 import goldy as G
+    from paper_2409_02227_gb300 import workloads as wl
+    l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
+    full_lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    n_sets = len(wl.scaling_study_shapes())
+    rows, summary = [], {}
+    geo = lambda xs: math.exp(sum(math.log(x) for x in xs) / len(xs))
+    for req, label in SCALING_PARTITIONS:
+        part = G.goldy_partition_create(req, 16)
+        sm, streams = G.goldy_partition_query(part, 16)
+        path = scaling_lut_path(sm)
+        tuned = G.goldy_lut_load(path) if os.path.exists(path) else None
+        for i in range(n_sets):
+            st = wl.make_scaling_set(i)
+            descs = [G.desc(x.M, x.N, x.K, x.out_dtype) for x in st.specs]
+            in_bytes = sum(2 * x.M * x.K + 2 * x.K * x.N for x in st.specs)
+            copies = min(16, max(2, math.ceil(2 * l2 / in_bytes)))
+            base_a = [a.cuda() for a in st.a]
+            base_b = [b.cuda() for b in st.b]
+            cdt = [torch.bfloat16 if x.out_dtype == 0 else torch.float32 for x in st.specs]
+            bufs = []
+            for r in range(copies):
+                A = base_a if r == 0 else [a.clone() for a in base_a]
+                B = base_b if r == 0 else [b.clone() for b in base_b]
+                C = [torch.empty((x.M, x.N), dtype=d, device="cuda") for x, d in zip(st.specs, cdt)]
+                bufs.append((A, B, C))
+            torch.cuda.synchronize()
+            pols = [("default", full_lut if tuned is None else tuned, G.GOLDY_PLAN_DEFAULT),
+                    ("sequential", full_lut if tuned is None else tuned, G.GOLDY_PLAN_SEQUENTIAL),
+                    ("goldyloc_whole_gpu_table", full_lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)]
+            if tuned is not None:
+                pols.append(("goldyloc", tuned, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED))
+            us = {}
+            for name, lut, flags in pols:
+                sched = G.goldy_plan(descs, lut, flags)
+                _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
+                ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+                torch.cuda.synchronize()
+                execs = [G.goldy_exec_create(sched, [a.data_ptr() for a in A], [b.data_ptr() for b in B],
+                                             [c.data_ptr() for c in C], ws.data_ptr(), ws_bytes,
+                                             streams[:max(1, ms)]) for A, B, C in bufs]
+                est = G.goldy_exec_time(execs, 2 * copies, copies) * 1e3
+                reps = int(min(2000, max(3 * copies, 20000.0 / max(est, 1.0))))
+                us[name] = G.goldy_exec_time(execs, 0, reps) * 1e3
+                del execs, ws
+            if G.goldy_device_error(clear=True) != 0:
+                raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
+            x = st.specs[0]
+            row = {"partition": label, "sms": sm, "set": st.name, "gemm": [x.M, x.N, x.K, x.out_dtype],
+                   "us": us}
+            rows.append(row)
+            del bufs, base_a, base_b, st
+            torch.cuda.empty_cache()
+        mine = [r for r in rows if r["partition"] == label]
+        best = "goldyloc" if tuned is not None else "goldyloc_whole_gpu_table"
+        summary[label] = {
+            "sms": sm, "table": path if tuned is not None else "whole-GPU table (no partition table found)",
+            "geomean_speedup_vs_default": geo([r["us"]["default"] / r["us"][best] for r in mine]),
+            "geomean_speedup_vs_sequential": geo([r["us"]["sequential"] / r["us"][best] for r in mine]),
+            "geomean_speedup_whole_gpu_table_vs_default": geo([r["us"]["default"] / r["us"]["goldyloc_whole_gpu_table"]
+                                                               for r in mine]),
+            "sets_faster_than_default": sum(r["us"]["default"] > r["us"][best] for r in mine), "sets": len(mine)}
+        print(label, json.dumps(summary[label]), flush=True)
+        del part
+    with open(args.scaling_study, "w") as f:
+        json.dump({"rows": rows, "summary": summary}, f, indent=1)
     return 0
 
 
@@ -690,6 +799,8 @@ def main(argv=None):
         return run_reference(args, world, rank)
     if args.report:
         return run_report(args, local)
+    if args.scaling_study:
+        return run_scaling_study(args, local)
     return run_gpu(args, world, rank, local)
 
 

@@ -161,6 +161,50 @@ goldy_status goldy_bucket_key(const goldy_gemm_desc* d, uint32_t* key);
 goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const goldy_lut* lut,
                         int flags, goldy_schedule** out);
 
+/* ---- logistic-regression CD predictor (Sec. 4.3, Eq. 1) -----------------
+ * The paper predicts each GEMM's preferred CD with a multi-class logistic
+ * regression trained offline once per GPU.  Features (GOLDY_LR_FEATURES, in
+ * this order): M, N, K, then for each CD class c in (1, 2, 4, 8, 16) three
+ * numbers of the table's GO-Kernel for the GEMM's bucket at c: its CTAs of
+ * work (output tiles x split-K slices; two CTAs per tile for a CTA-pair
+ * kernel), its CTAs resident per SM, and its waves (CTAs of work over
+ * CTAs/SM x sm_count / grid-cap divisor, rounded up).  The model min-max
+ * normalises them ((x - lo) / (hi - lo), 0 where hi == lo), scores each
+ * class s_c = b_c + sum_j W[c][j] x_j (in j order, doubles, no fused
+ * multiply-add), and predicts the class of largest score (= largest Eq. 1
+ * probability; ties to the smaller CD).
+ * Model file (little-endian): magic "GOLDYLRM", u32 version = 1, u32 feature
+ * count = 18, u32 class count = 5, u32 SM count (> 0), 8 zero bytes; then
+ * f64 lo[18], hi[18], W[5][18] (class-major), b[5]; all finite, hi >= lo.
+ * GOLDY_ERR_LUT if malformed.  The library owns the object. */
+#define GOLDY_LR_FEATURES 18
+typedef struct goldy_predictor goldy_predictor;
+goldy_status goldy_predictor_load(const char* path, goldy_predictor** out);
+goldy_status goldy_predictor_from_memory(const void* data, size_t bytes, goldy_predictor** out);
+void goldy_predictor_free(goldy_predictor* p);
+
+/* The table entry a GEMM plans with (its bucket, or the nearest stored one):
+ * preferred CD and the variant per CD class. */
+goldy_status goldy_lut_lookup(const goldy_lut* lut, const goldy_gemm_desc* d, int* pref_cd, int variants[5]);
+
+/* The predictor's raw (unnormalised) features of one GEMM against a table,
+ * for an SM count (> 0).  Used to build the training set. */
+goldy_status goldy_lr_features(const goldy_gemm_desc* d, const goldy_lut* lut, int sm_count,
+                               double out[GOLDY_LR_FEATURES]);
+
+/* Predicted preferred CD (1, 2, 4, 8 or 16) of one GEMM; probs (may be null)
+ * receives Eq. 1's probability per CD class. */
+goldy_status goldy_predict_cd(const goldy_predictor* p, const goldy_lut* lut, const goldy_gemm_desc* d,
+                              int* cd, double probs[5]);
+
+/* goldy_plan with the predictor (may be null: same as goldy_plan) supplying
+ * the preferred CDs under GOLDY_PLAN_AUTO: a bucket's preference is the
+ * smallest prediction over its GEMMs, and the CD run is still
+ * min(preference, GEMMs available).  Kernels still come from the table.  The
+ * forced policies ignore the predictor. */
+goldy_status goldy_plan_ex(const goldy_gemm_desc* descs, int n, const goldy_lut* lut,
+                           const goldy_predictor* predictor, int flags, goldy_schedule** out);
+
 /* Explicit schedule (used by the offline profiler and for measuring any
  * chosen schedule): GEMM i runs in group group_of[i] (groups are run in
  * increasing order, ids 0 .. n_groups-1 all used), with variant
@@ -248,6 +292,34 @@ goldy_status goldy_exec_create(const goldy_schedule* s, const void* const* A, co
 /* Enqueue a prepared run (asynchronous, no allocation). */
 goldy_status goldy_exec_launch(const goldy_exec* e);
 void goldy_exec_free(goldy_exec* e);
+
+/* Device time of prepared runs replayed back to back: `warmup` untimed
+ * replays, then `reps` replays timed by CUDA events on the first stream
+ * (replay k uses execs[k % n]: rotate copies of the inputs past the L2).  All
+ * n runs must share their first stream and partition.  Synchronises on the
+ * end event; *ms_per_rep = elapsed / reps.  Events live in the runs'
+ * partition, so this also times work inside an SM partition. */
+goldy_status goldy_exec_time(const goldy_exec* const* execs, int n, int warmup, int reps, float* ms_per_rep);
+
+/* ---- SM partitions (the paper's CU-partition study, Sec. 6.7) -----------
+ * A partition is a CUDA green context owning a subset of the GPU's SMs plus
+ * n_streams (1 .. GOLDY_MAX_STREAMS) non-blocking streams in it; kernels
+ * enqueued on those streams run on the partition's SMs only.  min_sms <= 0
+ * or >= the device's SMs gives the whole device as a partition; otherwise the
+ * driver rounds min_sms up to its partition granularity (query the actual
+ * count).  Passing a partition's streams to goldy_run / goldy_run_ex /
+ * goldy_exec_create / goldy_graph_create(_ex) / goldy_graph_launch runs the
+ * schedule inside the partition: grid caps are computed from the partition's
+ * SM count, and the library makes the partition's context current on the
+ * calling thread for the duration of each call (device memory of the
+ * device's primary context stays valid).  GOLDY_ERR_UNSUPPORTED if the
+ * driver has no green contexts or cannot split off such a partition.  Free
+ * every exec and graph that uses a partition before the partition. */
+typedef struct goldy_partition goldy_partition;
+goldy_status goldy_partition_create(int min_sms, int n_streams, goldy_partition** out);
+/* SM count, and the first n (<= n_streams) streams (CUstream handles). */
+goldy_status goldy_partition_query(const goldy_partition* p, int* sm_count, void** streams, int n);
+void goldy_partition_free(goldy_partition* p);
 
 /* Capture goldy_run(...) with these exact pointers into a CUDA graph, for
  * replay with one launch (the closest host-side analogue of the command

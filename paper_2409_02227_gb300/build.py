@@ -48,7 +48,7 @@ def _jobs(ptxas_verbose: bool):
     if ptxas_verbose:
         cu += ["-Xptxas", "-v"]
     jobs = []
-    jobs.append(("planner", ["g++", "-std=c++17", "-O2", "-fPIC", "-Wall", "-I", CSRC, "-I", INCLUDE,
+    jobs.append(("planner", ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fPIC", "-Wall", "-I", CSRC, "-I", INCLUDE,
                              "-c", os.path.join(CSRC, "planner.cpp")]))
     jobs.append(("runtime", cu + ["-c", os.path.join(CSRC, "runtime.cu")]))
     jobs.append(("noalloc", cu + ["-c", os.path.join(CSRC, "noalloc.cu")]))

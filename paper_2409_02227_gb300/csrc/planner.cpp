@@ -20,6 +20,7 @@
 //   slots    = member j of a group -> slot j mod CD
 //   kernel   = table's variant for the smallest CD class >= the group's CD
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <fstream>
@@ -160,6 +161,70 @@ extern "C" goldy_status goldy_lut_load(const char* path, goldy_lut** out) {
 
 extern "C" void goldy_lut_free(goldy_lut* lut) { delete lut; }
 
+// ---------------------------------------------------------------------------
+// Logistic-regression CD predictor (Sec. 4.3, Eq. 1)
+// ---------------------------------------------------------------------------
+struct goldy_predictor {
+  double lo[GOLDY_LR_FEATURES], hi[GOLDY_LR_FEATURES];
+  double W[5][GOLDY_LR_FEATURES], b[5];
+  uint32_t sm_count = 0;
+};
+
+static double rd_f64(const uint8_t* p) {
+  uint64_t u = 0;
+  for (int i = 7; i >= 0; --i) u = (u << 8) | p[i];
+  double d;
+  std::memcpy(&d, &u, sizeof d);
+  return d;
+}
+
+extern "C" goldy_status goldy_predictor_from_memory(const void* data, size_t bytes, goldy_predictor** out) {
+  if (!data || !out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  constexpr int nf = GOLDY_LR_FEATURES, nc = 5;
+  const uint8_t* p = static_cast<const uint8_t*>(data);
+  if (bytes < 32 || std::memcmp(p, "GOLDYLRM", 8) != 0) return fail(GOLDY_ERR_LUT, "predictor: bad magic");
+  if (rd32(p + 8) != 1 || rd32(p + 12) != uint32_t(nf) || rd32(p + 16) != uint32_t(nc))
+    return fail(GOLDY_ERR_LUT, "predictor: unsupported version or shape");
+  const uint32_t sm = rd32(p + 20);
+  if (sm == 0) return fail(GOLDY_ERR_LUT, "predictor: SM count is zero");
+  if (bytes != 32 + 8 * size_t(2 * nf + nc * nf + nc)) return fail(GOLDY_ERR_LUT, "predictor: bad size");
+  goldy_predictor* m = new (std::nothrow) goldy_predictor();
+  if (!m) return fail(GOLDY_ERR_NOMEM, "predictor: out of host memory");
+  m->sm_count = sm;
+  const uint8_t* q = p + 32;
+  bool bad = false;
+  auto next = [&]() {
+    const double v = rd_f64(q);
+    q += 8;
+    bad |= !std::isfinite(v);
+    return v;
+  };
+  for (int j = 0; j < nf; ++j) m->lo[j] = next();
+  for (int j = 0; j < nf; ++j) m->hi[j] = next();
+  for (int c = 0; c < nc; ++c)
+    for (int j = 0; j < nf; ++j) m->W[c][j] = next();
+  for (int c = 0; c < nc; ++c) m->b[c] = next();
+  for (int j = 0; j < nf && !bad; ++j) bad |= (m->hi[j] < m->lo[j]);
+  if (bad) {
+    delete m;
+    return fail(GOLDY_ERR_LUT, "predictor: non-finite value or hi below lo");
+  }
+  *out = m;
+  return ok();
+}
+
+extern "C" goldy_status goldy_predictor_load(const char* path, goldy_predictor** out) {
+  if (!path || !out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  std::ifstream f(path, std::ios::binary);
+  if (!f) return fail(GOLDY_ERR_LUT, std::string("predictor: cannot open ") + path);
+  std::vector<char> buf((std::istreambuf_iterator<char>(f)), std::istreambuf_iterator<char>());
+  return goldy_predictor_from_memory(buf.data(), buf.size(), out);
+}
+
+extern "C" void goldy_predictor_free(goldy_predictor* m) { delete m; }
+
 static uint32_t bucket_key(const goldy_gemm_desc& d) {
   return (uint32_t(floor_log2_u8(d.M)) << 24) | (uint32_t(floor_log2_u8(d.N)) << 16) |
          (uint32_t(floor_log2_u8(d.K)) << 8) | uint32_t(d.c_dtype & 0xFF);
@@ -185,6 +250,82 @@ static const LutEntry& lookup(const goldy_lut& lut, uint32_t key) {
     }
   }
   return lut.entries[best];
+}
+
+extern "C" goldy_status goldy_lut_lookup(const goldy_lut* lut, const goldy_gemm_desc* d, int* pref_cd,
+                                         int variants[5]) {
+  if (!lut || !d || !pref_cd || !variants) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  const LutEntry& e = lookup(*lut, bucket_key(*d));
+  *pref_cd = e.pref_cd;
+  for (int c = 0; c < 5; ++c) variants[c] = e.variant[c];
+  return ok();
+}
+
+// Features of one GEMM for the predictor (Sec. 4.3): M, N, K, then for each
+// CD class the table's GO-Kernel's CTAs of work (tiles x split-K slices, two
+// CTAs per tile for a CTA pair), CTAs resident per SM, and waves (CTAs of work
+// over the capped persistent grid, rounded up).
+static void lr_features(const goldy_gemm_desc& d, const LutEntry& e, int64_t sm_count,
+                        double x[GOLDY_LR_FEATURES]) {
+  x[0] = double(d.M);
+  x[1] = double(d.N);
+  x[2] = double(d.K);
+  for (int c = 0; c < 5; ++c) {
+    const Variant v = variant_of(e.variant[c]);
+    const KindInfo& k = kKinds[v.kind];
+    const int64_t per_tile = k.pair ? 2 : 1;
+    const int64_t split = k.pair ? 1 : v.split;
+    const int64_t ctas = ceil_div(d.M, tile_rows(k)) * ceil_div(d.N, tile_cols(k)) * split * per_tile;
+    const int64_t cap = std::max<int64_t>(per_tile, int64_t(k.ctas_per_sm) * sm_count / v.rc_div);
+    x[3 + 3 * c] = double(ctas);
+    x[4 + 3 * c] = double(k.ctas_per_sm);
+    x[5 + 3 * c] = double(ceil_div(ctas, cap));
+  }
+}
+
+extern "C" goldy_status goldy_lr_features(const goldy_gemm_desc* d, const goldy_lut* lut, int sm_count,
+                                          double out[GOLDY_LR_FEATURES]) {
+  if (!d || !lut || !out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  if (sm_count < 1) return fail(GOLDY_ERR_INVALID_ARG, "SM count must be positive");
+  goldy_status st = check_desc(*d, 0);
+  if (st != GOLDY_OK) return st;
+  lr_features(*d, lookup(*lut, bucket_key(*d)), sm_count, out);
+  return ok();
+}
+
+// Class index (0..4 for CD 1, 2, 4, 8, 16) of largest score; scores are
+// accumulated in a fixed order without contraction so that the decision is
+// reproducible bit for bit.
+static int lr_predict(const goldy_predictor& m, const double x[GOLDY_LR_FEATURES], double s[5]) {
+  int best = 0;
+  for (int c = 0; c < 5; ++c) {
+    double acc = m.b[c];
+    for (int j = 0; j < GOLDY_LR_FEATURES; ++j) {
+      const double xn = m.hi[j] > m.lo[j] ? (x[j] - m.lo[j]) / (m.hi[j] - m.lo[j]) : 0.0;
+      const double t = m.W[c][j] * xn;
+      acc = acc + t;
+    }
+    s[c] = acc;
+    if (c > 0 && s[c] > s[best]) best = c;
+  }
+  return best;
+}
+
+extern "C" goldy_status goldy_predict_cd(const goldy_predictor* m, const goldy_lut* lut, const goldy_gemm_desc* d,
+                                         int* cd, double probs[5]) {
+  if (!m || !lut || !d || !cd) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  goldy_status st = check_desc(*d, 0);
+  if (st != GOLDY_OK) return st;
+  double x[GOLDY_LR_FEATURES], s[5];
+  lr_features(*d, lookup(*lut, bucket_key(*d)), m->sm_count, x);
+  const int best = lr_predict(*m, x, s);
+  *cd = kCdClasses[best];
+  if (probs) {   // Eq. 1
+    double tot = 0.0;
+    for (int c = 0; c < 5; ++c) tot += (probs[c] = std::exp(s[c] - s[best]));
+    for (int c = 0; c < 5; ++c) probs[c] /= tot;
+  }
+  return ok();
 }
 
 // ---------------------------------------------------------------------------
@@ -240,6 +381,11 @@ static goldy_status new_schedule(const goldy_gemm_desc* descs, int n, goldy_sche
 
 extern "C" goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const goldy_lut* lut,
                                    int flags, goldy_schedule** out) {
+  return goldy_plan_ex(descs, n, lut, nullptr, flags, out);
+}
+
+extern "C" goldy_status goldy_plan_ex(const goldy_gemm_desc* descs, int n, const goldy_lut* lut,
+                                      const goldy_predictor* predictor, int flags, goldy_schedule** out) {
   if (!lut) return fail(GOLDY_ERR_LUT, "no lookup table");
   const int policy = flags & 0xF;
   const int forced = (flags >> 8) & 0xFF;
@@ -253,9 +399,16 @@ extern "C" goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const go
 
   std::vector<uint32_t> keys(n);
   std::vector<const LutEntry*> ent(n);
+  std::vector<int> pref(n);
   for (int i = 0; i < n; ++i) {
     keys[i] = bucket_key(descs[i]);
     ent[i] = &lookup(*lut, keys[i]);
+    pref[i] = ent[i]->pref_cd;
+    if (predictor && policy == GOLDY_PLAN_AUTO) {   // the trained model replaces the table's preference
+      double x[GOLDY_LR_FEATURES], sc[5];
+      lr_features(descs[i], *ent[i], predictor->sm_count, x);
+      pref[i] = kCdClasses[lr_predict(*predictor, x, sc)];
+    }
   }
 
   // (cd, members, class-cd override) triples; class-cd 0 means "use cd"
@@ -290,10 +443,11 @@ extern "C" goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const go
         const unsigned __int128 f =
             (unsigned __int128)2 * uint64_t(descs[i].M) * uint64_t(descs[i].N) * uint64_t(descs[i].K);
         if (it == blocks.end()) {
-          blocks.push_back({keys[i], f, {i}, ent[i]->pref_cd});
+          blocks.push_back({keys[i], f, {i}, pref[i]});
         } else {
           it->flops += f;
           it->members.push_back(i);
+          it->pref = std::min(it->pref, pref[i]);
         }
       }
       std::sort(blocks.begin(), blocks.end(), [](const Block& a, const Block& b) {

@@ -34,6 +34,7 @@ __device__ int g_device_error;   // kernels' error word (first failure wins)
 
 struct Runtime {
   int device = -1;
+  void* green = nullptr;   // green context the events were created under (null: the device's own)
   cudaEvent_t fork = nullptr;
   cudaEvent_t join[GOLDY_MAX_STREAMS] = {};
 };
@@ -349,6 +350,98 @@ goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream)
 }
 
 // Phase-trace buffer of the current goldy_run_ex call (null: off).
+// ---------------------------------------------------------------------------
+// SM partitions (CUDA green contexts).  A partition is a green context owning
+// a subset of the SMs; work on its streams runs on those SMs only.  Every
+// entry point that enqueues work makes the partition of its first stream
+// current for the duration of the call and sizes grids for its SM count.
+// ---------------------------------------------------------------------------
+struct GreenApi {
+  PFN_cuDeviceGet_v2000 device_get = nullptr;
+  PFN_cuDeviceGetDevResource_v12040 dev_resource = nullptr;
+  PFN_cuDevSmResourceSplitByCount_v12040 split = nullptr;
+  PFN_cuDevResourceGenerateDesc_v12040 gen_desc = nullptr;
+  PFN_cuGreenCtxCreate_v12040 create = nullptr;
+  PFN_cuGreenCtxDestroy_v12040 destroy = nullptr;
+  PFN_cuGreenCtxGetDevResource_v12040 ctx_resource = nullptr;
+  PFN_cuGreenCtxStreamCreate_v12050 stream_create = nullptr;
+  PFN_cuStreamDestroy_v4000 stream_destroy = nullptr;
+  PFN_cuStreamGetGreenCtx_v12040 stream_green = nullptr;
+  PFN_cuCtxFromGreenCtx_v12040 to_ctx = nullptr;
+  PFN_cuCtxPushCurrent_v4000 push = nullptr;
+  PFN_cuCtxPopCurrent_v4000 pop = nullptr;
+  bool ok = false;
+};
+
+const GreenApi& green_api() {
+  static GreenApi api = [] {
+    GreenApi a;
+    auto get = [](const char* name, int ver, void** fn) {
+      cudaDriverEntryPointQueryResult q;
+      return cudaGetDriverEntryPointByVersion(name, fn, ver, cudaEnableDefault, &q) == cudaSuccess &&
+             q == cudaDriverEntryPointSuccess && *fn;
+    };
+    bool ok = true;
+    ok &= get("cuDeviceGet", 2000, reinterpret_cast<void**>(&a.device_get));
+    ok &= get("cuDeviceGetDevResource", 12040, reinterpret_cast<void**>(&a.dev_resource));
+    ok &= get("cuDevSmResourceSplitByCount", 12040, reinterpret_cast<void**>(&a.split));
+    ok &= get("cuDevResourceGenerateDesc", 12040, reinterpret_cast<void**>(&a.gen_desc));
+    ok &= get("cuGreenCtxCreate", 12040, reinterpret_cast<void**>(&a.create));
+    ok &= get("cuGreenCtxDestroy", 12040, reinterpret_cast<void**>(&a.destroy));
+    ok &= get("cuGreenCtxGetDevResource", 12040, reinterpret_cast<void**>(&a.ctx_resource));
+    ok &= get("cuGreenCtxStreamCreate", 12050, reinterpret_cast<void**>(&a.stream_create));
+    ok &= get("cuStreamDestroy", 4000, reinterpret_cast<void**>(&a.stream_destroy));
+    ok &= get("cuStreamGetGreenCtx", 12040, reinterpret_cast<void**>(&a.stream_green));
+    ok &= get("cuCtxFromGreenCtx", 12040, reinterpret_cast<void**>(&a.to_ctx));
+    ok &= get("cuCtxPushCurrent", 4000, reinterpret_cast<void**>(&a.push));
+    ok &= get("cuCtxPopCurrent", 4000, reinterpret_cast<void**>(&a.pop));
+    a.ok = ok;
+    return a;
+  }();
+  return api;
+}
+
+// SMs the current run may use: the partition's when its streams belong to a
+// green context, else the device's (0).
+thread_local int t_sms = 0;
+
+// Makes the green context of `stream` (if it has one) current on this thread
+// until destroyed, and sets t_sms to its SM count.
+class PartitionScope {
+ public:
+  goldy_status enter(void* stream) {
+    green_ = nullptr;
+    if (!stream) return GOLDY_OK;
+    const GreenApi& g = green_api();
+    if (!g.ok) return GOLDY_OK;                  // no green contexts: every stream is the device's
+    CUgreenCtx gc = nullptr;
+    if (g.stream_green(static_cast<CUstream>(stream), &gc) != CUDA_SUCCESS || !gc) return GOLDY_OK;
+    CUcontext ctx = nullptr;
+    if (g.to_ctx(&ctx, gc) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuCtxFromGreenCtx failed");
+    CUdevResource res;
+    std::memset(&res, 0, sizeof(res));
+    if (g.ctx_resource(gc, &res, CU_DEV_RESOURCE_TYPE_SM) != CUDA_SUCCESS)
+      return fail(GOLDY_ERR_CUDA, "cuGreenCtxGetDevResource failed");
+    if (g.push(ctx) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuCtxPushCurrent failed");
+    green_ = gc;
+    saved_sms_ = t_sms;
+    t_sms = int(res.sm.smCount);
+    return GOLDY_OK;
+  }
+  void* green() const { return green_; }
+  ~PartitionScope() {
+    if (!green_) return;
+    CUcontext popped = nullptr;
+    green_api().pop(&popped);
+    t_sms = saved_sms_;
+  }
+
+ private:
+  void* green_ = nullptr;
+  int saved_sms_ = 0;
+};
+int sms(const DeviceState& d) { return t_sms > 0 ? std::min(t_sms, d.sm_count) : d.sm_count; }
+
 thread_local unsigned long long* t_trace = nullptr;
 thread_local size_t t_trace_ctas = 0;
 
@@ -377,8 +470,8 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   p.err = d.err_word;
 
   const Variant v = variant_of(gp.variant);
-  int64_t cap = std::max<int64_t>(1, int64_t(ctas) * d.sm_count / v.rc_div);
-  if (scale > 0.0) cap = std::min<int64_t>(int64_t(ctas) * d.sm_count, int64_t(double(cap) * scale));
+  int64_t cap = std::max<int64_t>(1, int64_t(ctas) * sms(d) / v.rc_div);
+  if (scale > 0.0) cap = std::min<int64_t>(int64_t(ctas) * sms(d), int64_t(double(cap) * scale));
   if (k.pair) {
     const unsigned grid = pair_grid(gp.units, cap);
     p.trace = trace_for(grid);
@@ -418,14 +511,14 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
     st = fill_slot(p, j, gp, A[members[j]], B[members[j]], C[members[j]], ws, int32_t(units));
     if (st != GOLDY_OK) return st;
     units += gp.units;
-    cap += std::max<int64_t>(1, int64_t(ctas) * d.sm_count / variant_of(gp.variant).rc_div);
+    cap += std::max<int64_t>(1, int64_t(ctas) * sms(d) / variant_of(gp.variant).rc_div);
   }
   if (units > int64_t(1) << 30) return fail(GOLDY_ERR_UNSUPPORTED, "too many tiles in one launch");
   p.n_gemms = count;
   p.total_units = int32_t(units);
   p.err = d.err_word;
   if (scale > 0.0) cap = int64_t(double(cap) * scale);
-  cap = std::min<int64_t>(cap, int64_t(ctas) * d.sm_count);
+  cap = std::min<int64_t>(cap, int64_t(ctas) * sms(d));
   if (k.pair) {
     const unsigned grid = pair_grid(units, cap);
     p.trace = trace_for(grid);
@@ -469,9 +562,10 @@ extern "C" goldy_status goldy_run(const goldy_schedule* s, const void* const* A,
 }
 
 namespace goldy {
-Runtime* new_runtime(int dev, goldy_status* st) {
+Runtime* new_runtime(int dev, void* green, goldy_status* st) {
   Runtime* rt = new Runtime();
   rt->device = dev;
+  rt->green = green;
   cudaError_t e = cudaEventCreateWithFlags(&rt->fork, cudaEventDisableTiming);
   for (int k = 0; k < GOLDY_MAX_STREAMS && e == cudaSuccess; ++k)
     e = cudaEventCreateWithFlags(&rt->join[k], cudaEventDisableTiming);
@@ -509,18 +603,21 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
   DeviceState* d = nullptr;
   goldy_status st = device_state(&d);
   if (st != GOLDY_OK) return st;
+  PartitionScope part;
+  st = part.enter(streams[0]);
+  if (st != GOLDY_OK) return st;
 
   Runtime* rt = own_rt;
   if (!rt) {
     goldy_schedule* ms = const_cast<goldy_schedule*>(s);
     int dev = 0;
     cudaGetDevice(&dev);
-    if (ms->rt && ms->rt->device != dev) {
+    if (ms->rt && (ms->rt->device != dev || ms->rt->green != part.green())) {
       runtime_release(ms->rt);
       ms->rt = nullptr;
     }
     if (!ms->rt) {
-      ms->rt = new_runtime(dev, &st);
+      ms->rt = new_runtime(dev, part.green(), &st);
       if (!ms->rt) return st;
     }
     rt = ms->rt;
@@ -650,6 +747,8 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
 struct goldy_exec {
   std::vector<Op> ops;
   Runtime* rt = nullptr;
+  CUcontext ctx = nullptr;   // the partition's context to make current while replaying (null: none)
+  cudaStream_t main = nullptr;
 };
 
 extern "C" goldy_status goldy_exec_create(const goldy_schedule* s, const void* const* A, const void* const* B,
@@ -661,10 +760,18 @@ extern "C" goldy_status goldy_exec_create(const goldy_schedule* s, const void* c
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  goldy_status st = GOLDY_OK;
+  if (!streams || n_streams < 1) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  PartitionScope part;
+  goldy_status st = part.enter(streams[0]);
+  if (st != GOLDY_OK) return st;
   goldy_exec* x = new (std::nothrow) goldy_exec();
   if (!x) return fail(GOLDY_ERR_NOMEM, "out of host memory");
-  x->rt = new_runtime(dev, &st);
+  if (part.green() && green_api().to_ctx(&x->ctx, static_cast<CUgreenCtx>(part.green())) != CUDA_SUCCESS) {
+    delete x;
+    return fail(GOLDY_ERR_CUDA, "cuCtxFromGreenCtx failed");
+  }
+  x->main = static_cast<cudaStream_t>(streams[0]);
+  x->rt = new_runtime(dev, part.green(), &st);
   if (!x->rt) {
     delete x;
     return st;
@@ -684,10 +791,50 @@ extern "C" goldy_status goldy_exec_create(const goldy_schedule* s, const void* c
 
 extern "C" goldy_status goldy_exec_launch(const goldy_exec* x) {
   if (!x) return fail(GOLDY_ERR_INVALID_ARG, "null exec");
+  if (x->ctx && green_api().push(x->ctx) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuCtxPushCurrent failed");
+  cudaError_t e = cudaSuccess;
   for (const Op& op : x->ops) {
-    cudaError_t e = replay(op);
-    if (e != cudaSuccess) return cuda_fail(e, "goldy_exec_launch");
+    e = replay(op);
+    if (e != cudaSuccess) break;
   }
+  if (x->ctx) {
+    CUcontext popped = nullptr;
+    green_api().pop(&popped);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "goldy_exec_launch");
+  return ok();
+}
+
+extern "C" goldy_status goldy_exec_time(const goldy_exec* const* execs, int n, int warmup, int reps,
+                                        float* ms_per_rep) {
+  if (!execs || n < 1 || warmup < 0 || reps < 1 || !ms_per_rep) return fail(GOLDY_ERR_INVALID_ARG, "bad argument");
+  for (int i = 0; i < n; ++i)
+    if (!execs[i] || execs[i]->ctx != execs[0]->ctx || execs[i]->main != execs[0]->main)
+      return fail(GOLDY_ERR_INVALID_ARG, "prepared runs must share their context and first stream");
+  const goldy_exec* x0 = execs[0];
+  if (x0->ctx && green_api().push(x0->ctx) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuCtxPushCurrent failed");
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  cudaError_t e = cudaEventCreate(&e0);
+  if (e == cudaSuccess) e = cudaEventCreate(&e1);
+  for (int k = 0; k < warmup && e == cudaSuccess; ++k)
+    for (const Op& op : execs[k % n]->ops)
+      if ((e = replay(op)) != cudaSuccess) break;
+  if (e == cudaSuccess) e = cudaEventRecord(e0, x0->main);
+  for (int k = 0; k < reps && e == cudaSuccess; ++k)
+    for (const Op& op : execs[k % n]->ops)
+      if ((e = replay(op)) != cudaSuccess) break;
+  if (e == cudaSuccess) e = cudaEventRecord(e1, x0->main);
+  if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+  float ms = 0.f;
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  if (x0->ctx) {
+    CUcontext popped = nullptr;
+    green_api().pop(&popped);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "goldy_exec_time");
+  *ms_per_rep = ms / float(reps);
   return ok();
 }
 
@@ -714,6 +861,9 @@ extern "C" goldy_status goldy_graph_create_ex(const goldy_schedule* s, const voi
                                               goldy_graph** out) {
   if (!out || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
   *out = nullptr;
+  PartitionScope part;
+  goldy_status pst = part.enter(streams[0]);
+  if (pst != GOLDY_OK) return pst;
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   cudaError_t e = cudaStreamBeginCapture(main, cudaStreamCaptureModeThreadLocal);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamBeginCapture");
@@ -741,6 +891,9 @@ extern "C" goldy_status goldy_graph_create_ex(const goldy_schedule* s, const voi
 
 extern "C" goldy_status goldy_graph_launch(const goldy_graph* g, void* stream) {
   if (!g) return fail(GOLDY_ERR_INVALID_ARG, "null graph");
+  PartitionScope part;
+  goldy_status pst = part.enter(stream);
+  if (pst != GOLDY_OK) return pst;
   cudaError_t e = cudaGraphLaunch(g->exec, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
   return ok();
@@ -794,3 +947,86 @@ goldy_status launch_planned_gemm(const GemmPlan& gp, const void* A, const void* 
   return launch_gemm(*d, gp, A, B, C, ws, static_cast<cudaStream_t>(stream));
 }
 }  // namespace goldy
+
+// ---------------------------------------------------------------------------
+// SM partitions
+// ---------------------------------------------------------------------------
+struct goldy_partition {
+  CUgreenCtx ctx = nullptr;
+  int sm_count = 0;
+  std::vector<CUstream> streams;
+};
+
+extern "C" void goldy_partition_free(goldy_partition* p) {
+  if (!p) return;
+  const GreenApi& g = green_api();
+  for (CUstream st : p->streams)
+    if (st) g.stream_destroy(st);
+  if (p->ctx) g.destroy(p->ctx);
+  delete p;
+}
+
+extern "C" goldy_status goldy_partition_create(int min_sms, int n_streams, goldy_partition** out) {
+  if (!out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  if (n_streams < 1 || n_streams > GOLDY_MAX_STREAMS) return fail(GOLDY_ERR_INVALID_ARG, "stream count out of range");
+  const GreenApi& g = green_api();
+  if (!g.ok) return fail(GOLDY_ERR_UNSUPPORTED, "green contexts are not available from this driver");
+  int dev = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
+  ce = cudaFree(nullptr);   // the primary context must exist before a green context retains it
+  if (ce != cudaSuccess) return cuda_fail(ce, "cudaFree(0)");
+  CUdevice cu = 0;
+  if (g.device_get(&cu, dev) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuDeviceGet failed");
+  CUdevResource all;
+  std::memset(&all, 0, sizeof(all));
+  if (g.dev_resource(cu, &all, CU_DEV_RESOURCE_TYPE_SM) != CUDA_SUCCESS)
+    return fail(GOLDY_ERR_CUDA, "cuDeviceGetDevResource failed");
+  CUdevResource part;
+  std::memset(&part, 0, sizeof(part));
+  if (min_sms <= 0 || unsigned(min_sms) >= all.sm.smCount) {
+    part = all;                                   // the whole device, as a partition
+  } else {
+    unsigned groups = 1;
+    CUdevResource rest;
+    std::memset(&rest, 0, sizeof(rest));
+    if (g.split(&part, &groups, &all, &rest, 0, unsigned(min_sms)) != CUDA_SUCCESS || groups != 1)
+      return fail(GOLDY_ERR_UNSUPPORTED, "cannot split off a partition of " + std::to_string(min_sms) + " SMs");
+  }
+  CUdevResourceDesc desc = nullptr;
+  if (g.gen_desc(&desc, &part, 1) != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuDevResourceGenerateDesc failed");
+  goldy_partition* p = new (std::nothrow) goldy_partition();
+  if (!p) return fail(GOLDY_ERR_NOMEM, "out of host memory");
+  if (g.create(&p->ctx, desc, cu, CU_GREEN_CTX_DEFAULT_STREAM) != CUDA_SUCCESS) {
+    p->ctx = nullptr;
+    goldy_partition_free(p);
+    return fail(GOLDY_ERR_CUDA, "cuGreenCtxCreate failed");
+  }
+  CUdevResource got;
+  std::memset(&got, 0, sizeof(got));
+  if (g.ctx_resource(p->ctx, &got, CU_DEV_RESOURCE_TYPE_SM) != CUDA_SUCCESS) {
+    goldy_partition_free(p);
+    return fail(GOLDY_ERR_CUDA, "cuGreenCtxGetDevResource failed");
+  }
+  p->sm_count = int(got.sm.smCount);
+  p->streams.assign(size_t(n_streams), nullptr);
+  for (int k = 0; k < n_streams; ++k) {
+    if (g.stream_create(&p->streams[size_t(k)], p->ctx, CU_STREAM_NON_BLOCKING, 0) != CUDA_SUCCESS) {
+      p->streams[size_t(k)] = nullptr;
+      goldy_partition_free(p);
+      return fail(GOLDY_ERR_CUDA, "cuGreenCtxStreamCreate failed");
+    }
+  }
+  *out = p;
+  return ok();
+}
+
+extern "C" goldy_status goldy_partition_query(const goldy_partition* p, int* sm_count, void** streams, int n) {
+  if (!p) return fail(GOLDY_ERR_INVALID_ARG, "null partition");
+  if (n < 0 || n > int(p->streams.size()) || (n > 0 && !streams))
+    return fail(GOLDY_ERR_INVALID_ARG, "stream count out of range");
+  if (sm_count) *sm_count = p->sm_count;
+  for (int k = 0; k < n; ++k) streams[k] = p->streams[size_t(k)];
+  return ok();
+}

@@ -16,6 +16,8 @@ from typing import List, Optional, Sequence, Tuple
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libgoldy.so")
 DEFAULT_LUT = os.path.join(_HERE, "data", "goldy_lut.bin")
+DEFAULT_PREDICTOR = os.path.join(_HERE, "data", "goldy_lr.bin")
+LR_FEATURES = 18
 
 GOLDY_OK = 0
 GOLDY_ERR_INVALID_ARG = 1
@@ -92,6 +94,13 @@ def _load():
         "goldy_lut_free": ([P], None),
         "goldy_bucket_key": ([DP, ctypes.POINTER(U32)], I),
         "goldy_plan": ([DP, I, P, I, PP], I),
+        "goldy_plan_ex": ([DP, I, P, P, I, PP], I),
+        "goldy_predictor_load": ([ctypes.c_char_p, PP], I),
+        "goldy_predictor_from_memory": ([P, SZ, PP], I),
+        "goldy_predictor_free": ([P], None),
+        "goldy_lut_lookup": ([P, DP, IP, IP], I),
+        "goldy_lr_features": ([DP, P, I, ctypes.POINTER(ctypes.c_double)], I),
+        "goldy_predict_cd": ([P, P, DP, IP, ctypes.POINTER(ctypes.c_double)], I),
         "goldy_schedule_build": ([DP, I, IP, IP, IP, I, PP], I),
         "goldy_schedule_query": ([P, IP, IP, IP, ctypes.POINTER(SZ)], I),
         "goldy_schedule_entry": ([P, I, IP, IP, IP, IP], I),
@@ -104,6 +113,10 @@ def _load():
         "goldy_graph_launch": ([P, P], I),
         "goldy_exec_create": ([P, PP, PP, PP, P, SZ, PP, I, ctypes.POINTER(goldy_run_opts), PP], I),
         "goldy_exec_launch": ([P], I),
+        "goldy_exec_time": ([PP, I, I, I, ctypes.POINTER(ctypes.c_float)], I),
+        "goldy_partition_create": ([I, I, PP], I),
+        "goldy_partition_query": ([P, IP, PP, I], I),
+        "goldy_partition_free": ([P], None),
         "goldy_exec_free": ([P], None),
         "goldy_graph_free": ([P], None),
         "goldy_gemm_noalloc": ([DP, I, P, P, P, P], I),
@@ -168,12 +181,20 @@ class Lut(_Handle):
     _free = staticmethod(lambda p: _lib.goldy_lut_free(p))
 
 
+class Predictor(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_predictor_free(p))
+
+
 class Schedule(_Handle):
     _free = staticmethod(lambda p: _lib.goldy_schedule_free(p))
 
 
 class Graph(_Handle):
     _free = staticmethod(lambda p: _lib.goldy_graph_free(p))
+
+
+class Partition(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_partition_free(p))
 
 
 class Exec(_Handle):
@@ -222,6 +243,47 @@ def goldy_plan(descs: Sequence[goldy_gemm_desc], lut: Lut, flags: int = GOLDY_PL
     _check(_lib.goldy_plan(_descs(descs), len(descs), lut.ptr if lut else None, int(flags),
                            ctypes.byref(out)), "goldy_plan")
     return Schedule(out)
+
+
+def goldy_plan_ex(descs: Sequence[goldy_gemm_desc], lut: Lut, predictor: Optional[Predictor],
+                  flags: int = GOLDY_PLAN_AUTO) -> Schedule:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_plan_ex(_descs(descs), len(descs), lut.ptr if lut else None,
+                              predictor.ptr if predictor else None, int(flags), ctypes.byref(out)), "goldy_plan_ex")
+    return Schedule(out)
+
+
+def goldy_predictor_load(path: str = DEFAULT_PREDICTOR) -> Predictor:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_predictor_load(path.encode(), ctypes.byref(out)), "goldy_predictor_load")
+    return Predictor(out)
+
+
+def goldy_predictor_from_memory(data: bytes) -> Predictor:
+    out = ctypes.c_void_p()
+    buf = ctypes.create_string_buffer(bytes(data), len(data))
+    _check(_lib.goldy_predictor_from_memory(buf, len(data), ctypes.byref(out)), "goldy_predictor_from_memory")
+    return Predictor(out)
+
+
+def goldy_lut_lookup(lut: Lut, d: goldy_gemm_desc) -> Tuple[int, List[int]]:
+    pref = ctypes.c_int()
+    vs = (ctypes.c_int * 5)()
+    _check(_lib.goldy_lut_lookup(lut.ptr, ctypes.byref(d), ctypes.byref(pref), vs), "goldy_lut_lookup")
+    return pref.value, list(vs)
+
+
+def goldy_lr_features(d: goldy_gemm_desc, lut: Lut, sm_count: int) -> List[float]:
+    out = (ctypes.c_double * LR_FEATURES)()
+    _check(_lib.goldy_lr_features(ctypes.byref(d), lut.ptr, int(sm_count), out), "goldy_lr_features")
+    return list(out)
+
+
+def goldy_predict_cd(p: Predictor, lut: Lut, d: goldy_gemm_desc) -> Tuple[int, List[float]]:
+    cd = ctypes.c_int()
+    probs = (ctypes.c_double * 5)()
+    _check(_lib.goldy_predict_cd(p.ptr, lut.ptr, ctypes.byref(d), ctypes.byref(cd), probs), "goldy_predict_cd")
+    return cd.value, list(probs)
 
 
 def goldy_schedule_build(descs: Sequence[goldy_gemm_desc], group_of: Sequence[int],
@@ -323,6 +385,28 @@ def goldy_exec_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequen
                                   int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o),
                                   ctypes.byref(out)), "goldy_exec_create")
     return Exec(out)
+
+
+def goldy_exec_time(execs: Sequence[Exec], warmup: int, reps: int) -> float:
+    """Milliseconds per replay (see include/goldy.h)."""
+    arr = (ctypes.c_void_p * len(execs))(*[e.ptr for e in execs])
+    ms = ctypes.c_float()
+    _check(_lib.goldy_exec_time(arr, len(execs), int(warmup), int(reps), ctypes.byref(ms)), "goldy_exec_time")
+    return ms.value
+
+
+def goldy_partition_create(min_sms: int, n_streams: int = 16) -> Partition:
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_partition_create(int(min_sms), int(n_streams), ctypes.byref(out)), "goldy_partition_create")
+    return Partition(out)
+
+
+def goldy_partition_query(p: Partition, n: int = 0) -> Tuple[int, List[int]]:
+    """(SM count, the first n stream handles as integers)."""
+    sm = ctypes.c_int()
+    arr = (ctypes.c_void_p * max(1, n))()
+    _check(_lib.goldy_partition_query(p.ptr, ctypes.byref(sm), arr, int(n)), "goldy_partition_query")
+    return sm.value, [int(arr[k] or 0) for k in range(n)]
 
 
 def goldy_exec_launch(e: Exec) -> None:

@@ -161,6 +161,50 @@ def sweep_specs(j: int) -> Tuple[int, List[GemmSpec], torch.Generator]:
     return seed, specs, gen
 
 
+def predictor_dataset_shapes(total: int = 1072, seed: int = 5000) -> List[Tuple[int, int, int, int]]:
+    """Distinct GEMM shapes (M, N, K, out dtype) for the CD predictor's
+    training set: those of the fixed sets and of the 64 randomized sets first,
+    then seeded log-uniform draws over the same ranges (M in [16, 4096]; N, K
+    multiples of 64 in [256, 8192]; bf16 or fp32 out) up to `total`."""
+    out: List[Tuple[int, int, int, int]] = []
+    seen = set()
+
+    def add(t):
+        if t not in seen and len(out) < total:
+            seen.add(t)
+            out.append(t)
+
+    for name in FIXED_CONFIGS:
+        for s in config_specs(name)[1]:
+            add((s.M, s.N, s.K, s.out_dtype))
+    for j in range(SWEEP_SETS):
+        for s in sweep_specs(j)[1]:
+            add((s.M, s.N, s.K, s.out_dtype))
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed)
+    while len(out) < total:
+        M = min(max(int(round(_log_uniform(gen, 16, 4096))), 16), 4096)
+        N = min(max(64 * int(round(_log_uniform(gen, 256, 8192) / 64)), 256), 8192)
+        K = min(max(64 * int(round(_log_uniform(gen, 256, 8192) / 64)), 256), 8192)
+        o = int(torch.randint(0, 2, (1,), generator=gen)[0])
+        add((M, N, K, DTYPE_BF16 if o == 0 else DTYPE_F32))
+    return out
+
+
+def scaling_study_shapes(stride: int = 16) -> List[Tuple[int, int, int, int]]:
+    """GEMM shapes of the GPU-scaling study (every `stride`-th shape of the
+    predictor's training set; each runs as a set of 4 equal GEMMs, CD 4)."""
+    return predictor_dataset_shapes()[::stride]
+
+
+def make_scaling_set(i: int, copies: int = 4) -> GemmSet:
+    """Set i of the GPU-scaling study: `copies` equal GEMMs, U[-1, 1] inputs,
+    seed 3000 + i."""
+    M, N, K, out = scaling_study_shapes()[i]
+    specs = [GemmSpec(M, N, K, out, "uniform", 1.0) for _ in range(copies)]
+    return materialize(f"scaling_{i:02d}", 3000 + i, specs)
+
+
 def make_sweep_set(j: int) -> GemmSet:
     seed, specs, gen = sweep_specs(j)
     return materialize(f"sweep_{j:02d}", seed, specs, gen)

@@ -151,3 +151,39 @@ def test_bucket_key_matches_reference():
         d = G.desc(M, N, K, c, lda=max(8, (K + 7) // 8 * 8), ldb=max(8, (N + 7) // 8 * 8), ldc=max(N, 1))
         lm, ln, lk, out = pr.bucket_key(M, N, K, c)
         assert G.goldy_bucket_key(d) == (lm << 24) | (ln << 16) | (lk << 8) | out
+
+
+def test_partition_and_exec_error_paths():
+    # no GPU here: creating a partition fails with a status, never a crash
+    with pytest.raises(G.GoldyError) as ei:
+        G.goldy_partition_create(38, 4)
+    assert ei.value.status in (G.GOLDY_ERR_UNSUPPORTED, G.GOLDY_ERR_CUDA)
+    lib = G._lib
+    import ctypes
+    out = ctypes.c_void_p()
+    assert lib.goldy_partition_create(38, 0, ctypes.byref(out)) == G.GOLDY_ERR_INVALID_ARG
+    assert lib.goldy_partition_create(38, 17, ctypes.byref(out)) == G.GOLDY_ERR_INVALID_ARG
+    assert lib.goldy_partition_create(38, 4, None) == G.GOLDY_ERR_INVALID_ARG
+    sm = ctypes.c_int()
+    assert lib.goldy_partition_query(None, ctypes.byref(sm), None, 0) == G.GOLDY_ERR_INVALID_ARG
+    lib.goldy_partition_free(None)
+    ms = ctypes.c_float()
+    assert lib.goldy_exec_time(None, 1, 0, 1, ctypes.byref(ms)) == G.GOLDY_ERR_INVALID_ARG
+    assert lib.goldy_exec_launch(None) == G.GOLDY_ERR_INVALID_ARG
+    lib.goldy_exec_free(None)
+
+
+def test_packaged_tables_and_predictor_load():
+    import glob
+    import os
+    from oracle import planner_ref as pr
+    from oracle import predictor_ref as P
+    paths = [G.DEFAULT_LUT] + sorted(glob.glob(os.path.join(os.path.dirname(G.DEFAULT_LUT), "scaling", "*.bin")))
+    assert len(paths) >= 4
+    for p in paths:
+        data = open(p, "rb").read()
+        G.goldy_lut_from_memory(data)
+        pr.parse_lut(data)
+    m = open(G.DEFAULT_PREDICTOR, "rb").read()
+    G.goldy_predictor_from_memory(m)
+    assert P.parse_model(m).sm_count == 152

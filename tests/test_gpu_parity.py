@@ -322,3 +322,20 @@ def test_sweep_sets_through_the_planner(cuda_ok, j):
     for i, s in enumerate(st.specs):
         rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(6, s.M))]))
         check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} gemm {i} {s.M}x{s.N}x{s.K}")
+
+
+@pytest.mark.parametrize("j", [0, 8, 33])
+def test_sweep_sets_through_the_predictor_plan(cuda_ok, j):
+    # sets whose schedule changes when the trained CD predictor (Eq. 1)
+    # supplies the preferences: sampled rows of every GEMM vs the oracle
+    st = wl.make_sweep_set(j)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    lut = G.goldy_lut_load(G.DEFAULT_LUT)
+    sched = G.goldy_plan_ex(descs, lut, G.goldy_predictor_load(), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    L = Launch(sched, st.a, st.b, [s.out_dtype for s in st.specs])
+    L.run()
+    got = L.results()
+    rng = np.random.default_rng(100 + j)
+    for i, s in enumerate(st.specs):
+        rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(6, s.M))]))
+        check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} (predictor plan) gemm {i} {s.M}x{s.N}x{s.K}")

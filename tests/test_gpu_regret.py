@@ -6,7 +6,9 @@ each GEMM with the table's GO-Kernel for that group size, is measured on the
 GPU; the oracle's brute-force search (oracle/schedule.py) then finds the best
 split into consecutive groups under those times, and the planner's own
 schedule is timed directly.  The regret (planner / best - 1) must stay small;
-the paper reports its predictor within 3% geomean of its Oracle.  Results are
+the paper reports its predictor within 3% geomean of its Oracle.  The plan
+with the trained logistic-regression predictor (Eq. 1) is timed the same way.
+Results are
 also written to gpurun_out/regret.json when that folder exists."""
 import json
 import math
@@ -78,12 +80,24 @@ def test_planner_regret_vs_exhaustive_oracle(cuda_ok, name):
     torch.cuda.synchronize()
     t_plan = r.timed(60)[0] / 60 * 1e3
     del r
+    # the same planner with the trained CD predictor supplying the preferences
+    t_lr = None
+    if os.path.exists(G.DEFAULT_PREDICTOR):
+        plan_lr = G.goldy_plan_ex(descs, G.goldy_lut_from_memory(lut_bytes), G.goldy_predictor_load(),
+                                  G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+        r = bench.SetRunner(st, plan_lr, 4)
+        for k in range(5):
+            r.launch(k)
+        torch.cuda.synchronize()
+        t_lr = r.timed(60)[0] / 60 * 1e3
+        del r
     # the oracle's schedule, timed the same way (its groups one after another)
     t_best = 0.0
     for blk in best.partition:
         t_best += cache[blk]
     regret = t_plan / t_best - 1.0
     record = {"set": name, "n": n, "planner_us": t_plan, "oracle_us": t_best, "regret": regret,
+              "planner_lr_us": t_lr, "regret_lr": None if t_lr is None else t_lr / t_best - 1.0,
               "oracle_partition": [list(b) for b in best.partition],
               "planner_groups": [e[0] for e in entries_plan],
               "subset_us": {",".join(map(str, k)): v for k, v in cache.items()}}
@@ -93,3 +107,5 @@ def test_planner_regret_vs_exhaustive_oracle(cuda_ok, name):
             f.write(json.dumps(record) + "\n")
     assert math.isfinite(regret)
     assert regret < 0.35, record
+    if t_lr is not None:
+        assert t_lr / t_best - 1.0 < 0.35, record
