@@ -60,6 +60,10 @@ def parse_args(argv=None):
                     help="how the prepared step is replayed: recorded plain launches or a CUDA graph")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--batched-study", default=None, metavar="FILE",
+                    help="heterogeneous strided-batched GEMM study (JSON to FILE)")
+    ap.add_argument("--corun-study", default=None, metavar="FILE",
+                    help="GEMM + element-wise add co-scheduling study (JSON to FILE)")
     ap.add_argument("--scaling-study", default=None, metavar="FILE",
                     help="GPU-scaling study inside SM partitions of 1/4, 1/2 and all of the GPU (JSON to FILE)")
     ap.add_argument("--report", default=None, metavar="FILE",
@@ -274,6 +278,11 @@ def run_reference(args, world, rank):
 
 
 # ----------------------------------------------------------------------------- GPU arm
+def c_shape(s):
+    """Shape of a GEMM's output (entries first for a strided batch)."""
+    return (s.M, s.N) if s.batch == 1 else (s.batch, s.M, s.N)
+
+
 class SetRunner:
     """R rotating device copies of one GEMM set, each with its run prepared
     once: a recorded prepared run (``replay="exec"``, plain launches) or a
@@ -298,7 +307,7 @@ class SetRunner:
         for r in range(copies):
             A = base_a if r == 0 else [a.clone() for a in base_a]
             B = base_b if r == 0 else [b.clone() for b in base_b]
-            C = [torch.empty((s.M, s.N), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
+            C = [torch.empty(c_shape(s), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
             self.copies.append((A, B, C))
         self.events = []
         self.runs = []
@@ -431,10 +440,10 @@ def e2e_measure(st, sched, steps):
     hA = [a.pin_memory() for a in st.a]
     hB = [b.pin_memory() for b in st.b]
     cdt = [torch.bfloat16 if s.out_dtype == 0 else torch.float32 for s in st.specs]
-    hC = [torch.empty((s.M, s.N), dtype=d).pin_memory() for s, d in zip(st.specs, cdt)]
+    hC = [torch.empty(c_shape(s), dtype=d).pin_memory() for s, d in zip(st.specs, cdt)]
     dA = [torch.empty_like(a, device="cuda") for a in st.a]
     dB = [torch.empty_like(b, device="cuda") for b in st.b]
-    dC = [torch.empty((s.M, s.N), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
+    dC = [torch.empty(c_shape(s), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
     main = streams[0]
     A = [a.data_ptr() for a in dA]
     B = [b.data_ptr() for b in dB]
@@ -474,7 +483,7 @@ def run_gpu(args, world, rank, local):
     from paper_2409_02227_gb300 import workloads as wl
 
     st = wl.make_config(args.config)
-    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
     lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
     launch_flag = G.GOLDY_PLAN_FUSED if args.launch == "fused" else 0
     sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | launch_flag)
@@ -484,7 +493,7 @@ def run_gpu(args, world, rank, local):
     single_launch = bool(launch_flag) and n_groups == 1 and len(kinds) == 1 and plan[0][3] >= len(descs)
     props = torch.cuda.get_device_properties(device)
     l2 = int(getattr(props, "L2_cache_size", 126 * 1024 * 1024))
-    in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
+    in_bytes = sum(s.batch * (2 * s.M * s.K + 2 * s.K * s.N) for s in st.specs)
     copies = max(2, math.ceil(2 * l2 / in_bytes))
 
     runner = SetRunner(st, sched, copies, replay=args.replay)
@@ -619,7 +628,7 @@ def time_policies(st, lut, copies, steps):
     """Makespan (us) of one set under each policy, timed like the main line."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
-    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
     out = {}
     predictor = G.goldy_predictor_load() if os.path.exists(G.DEFAULT_PREDICTOR) else None
     for name, flags in (("goldyloc", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED),
@@ -658,7 +667,7 @@ def run_report(args, local):
     for name, st in sets:
         if st is None:
             st = wl.make_sweep_set(int(name.split("_")[1]))
-        in_bytes = sum(2 * s.M * s.K + 2 * s.K * s.N for s in st.specs)
+        in_bytes = sum(s.batch * (2 * s.M * s.K + 2 * s.K * s.N) for s in st.specs)
         copies = max(2, math.ceil(2 * l2 / in_bytes))
         steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
         t = time_policies(st, lut, copies, steps)
@@ -792,6 +801,127 @@ def run_scaling_study(args, local):
     return 0
 
 
+def run_batched_study(args, local):
+    """Heterogeneous strided-batched GEMMs (Sec. 6.6): sets of 2 and 4
+    batched attention GEMMs over variable sequence lengths, under default
+    (isolation-tuned kernels, every B-GEMM on its own stream), sequential,
+    GO at CD = n, and GOLDYLOC; each configuration at its faster replay,
+    inputs rotated past the L2."""
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2409_02227_gb300 import goldy as G
+    from paper_2409_02227_gb300 import workloads as wl
+    l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
+    lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    rows = []
+    for members in (2, 4):
+        for i in range(16):
+            st = wl.make_batched_set(i, members)
+            descs = [G.desc(x.M, x.N, x.K, x.out_dtype, batch=x.batch) for x in st.specs]
+            in_bytes = sum(x.batch * (2 * x.M * x.K + 2 * x.K * x.N) for x in st.specs)
+            copies = min(16, max(2, math.ceil(2 * l2 / in_bytes)))
+            steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
+            us, plans = {}, {}
+            for name, flags in (("default", G.GOLDY_PLAN_DEFAULT), ("sequential", G.GOLDY_PLAN_SEQUENTIAL),
+                                ("go_all_concurrent", G.GOLDY_PLAN_GO | G.GOLDY_PLAN_FUSED),
+                                ("goldyloc", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
+                sched = G.goldy_plan(descs, lut, flags)
+                us[name], _ = time_schedule(st, sched, copies, steps)
+                plans[name] = [G.goldy_schedule_entry(sched, k) for k in range(len(descs))]
+            if G.goldy_device_error(clear=True) != 0:
+                raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
+            rows.append({"set": st.name, "members": members,
+                         "gemms": [[x.M, x.N, x.K, x.batch] for x in st.specs], "us": us,
+                         "goldyloc_plan": [{"group": g, "variant": G.goldy_variant_info_get(v)["name"], "cd": cd}
+                                           for g, v, _, cd in plans["goldyloc"]]})
+            print(st.name, {k: round(v, 2) for k, v in us.items()}, flush=True)
+            del st
+            torch.cuda.empty_cache()
+    geo = lambda xs: math.exp(sum(math.log(x) for x in xs) / len(xs))
+    summary = {}
+    for members in (2, 4):
+        sel = [r for r in rows if r["members"] == members]
+        summary[f"{members}P"] = {
+            "sets": len(sel),
+            "goldyloc_speedup_vs_default": geo([r["us"]["default"] / r["us"]["goldyloc"] for r in sel]),
+            "goldyloc_max_speedup_vs_default": max(r["us"]["default"] / r["us"]["goldyloc"] for r in sel),
+            "goldyloc_speedup_vs_sequential": geo([r["us"]["sequential"] / r["us"]["goldyloc"] for r in sel]),
+            "go_speedup_vs_default": geo([r["us"]["default"] / r["us"]["go_all_concurrent"] for r in sel])}
+    print(json.dumps(summary), flush=True)
+    with open(args.batched_study, "w") as f:
+        json.dump({"rows": rows, "summary": summary}, f, indent=1)
+    return 0
+
+
+def run_corun_study(args, local):
+    """GEMM + element-wise add (Sec. 8.1): each study GEMM co-scheduled with
+    an add over its output size under sequential, default (isolation-tuned
+    GEMM kernel and the add at once), GO (CD-2 GO-Kernel and a half-GPU add at
+    once) and GOLDYLOC (GO where the table marks co-running as paying, else
+    sequential).  Prepared runs, inputs rotated past the L2."""
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2409_02227_gb300 import goldy as G
+    from paper_2409_02227_gb300 import workloads as wl
+    l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
+    hbm, tf_burst, _, _ = peaks()
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    sp = [x.cuda_stream for x in streams]
+    rows = []
+    for i, (M, N, K, out) in enumerate(wl.scaling_study_shapes()):
+        td = torch.bfloat16 if out == G.GOLDY_BF16 else torch.float32
+        es = 2 if out == G.GOLDY_BF16 else 4
+        in_bytes = 2 * M * K + 2 * K * N + 2 * es * M * N
+        copies = min(16, max(2, math.ceil(2 * l2 / in_bytes)))
+        g = torch.Generator(device="cuda")
+        g.manual_seed(4000 + i)
+        bufs = []
+        for _ in range(copies):
+            bufs.append(((torch.rand((M, K), generator=g, device="cuda") - 0.5).to(torch.bfloat16),
+                         (torch.rand((K, N), generator=g, device="cuda") - 0.5).to(torch.bfloat16),
+                         torch.empty((M, N), dtype=td, device="cuda"),
+                         torch.randn(M * N, generator=g, device="cuda").to(td),
+                         torch.randn(M * N, generator=g, device="cuda").to(td),
+                         torch.empty(M * N, dtype=td, device="cuda")))
+        us, plan = {}, {}
+        for name, pol in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("default", G.GOLDY_PLAN_DEFAULT),
+                          ("go", G.GOLDY_PLAN_GO), ("goldyloc", G.GOLDY_PLAN_AUTO)):
+            c = G.goldy_corun_plan(G.desc(M, N, K, out), M * N, out, lut, pol)
+            conc, v, rc, ws_bytes = G.goldy_corun_query(c)
+            ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+            torch.cuda.synchronize()
+            execs = [G.goldy_corun_exec_create(c, A.data_ptr(), B.data_ptr(), C.data_ptr(), ws.data_ptr(), ws_bytes,
+                                               X.data_ptr(), Y.data_ptr(), Z.data_ptr(), sp)
+                     for A, B, C, X, Y, Z in bufs]
+            est = G.goldy_exec_time(execs, 2 * copies, copies) * 1e3
+            reps = int(min(4000, max(3 * copies, 20000.0 / max(est, 1.0))))
+            us[name] = G.goldy_exec_time(execs, 0, reps) * 1e3
+            plan[name] = {"concurrent": conc, "variant": G.goldy_variant_info_get(v)["name"], "add_rc_div": rc}
+            del execs, ws
+        if G.goldy_device_error(clear=True) != 0:
+            raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
+        flops = 2 * M * N * K
+        gemm_bytes = 2 * M * K + 2 * K * N + es * M * N
+        rows.append({"gemm": [M, N, K, out], "memory_bound_gemm": flops / gemm_bytes < ridge, "us": us,
+                     "plan": plan})
+        del bufs
+        torch.cuda.empty_cache()
+    geo = lambda xs: math.exp(sum(math.log(x) for x in xs) / len(xs)) if xs else None
+    summary = {}
+    for sub, sel in (("all", rows), ("memory_bound", [r for r in rows if r["memory_bound_gemm"]]),
+                     ("compute_bound", [r for r in rows if not r["memory_bound_gemm"]])):
+        summary[sub] = {"gemms": len(sel)}
+        for name in ("sequential", "go", "goldyloc"):
+            summary[sub][f"{name}_speedup_vs_default"] = geo([r["us"]["default"] / r["us"][name] for r in sel])
+        summary[sub]["goldyloc_co_runs"] = sum(r["plan"]["goldyloc"]["concurrent"] for r in sel)
+    print(json.dumps(summary), flush=True)
+    with open(args.corun_study, "w") as f:
+        json.dump({"rows": rows, "summary": summary}, f, indent=1)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     world, rank, local = dist_env()
@@ -801,6 +931,10 @@ def main(argv=None):
         return run_report(args, local)
     if args.scaling_study:
         return run_scaling_study(args, local)
+    if args.corun_study:
+        return run_corun_study(args, local)
+    if args.batched_study:
+        return run_batched_study(args, local)
     return run_gpu(args, world, rank, local)
 
 

@@ -55,16 +55,23 @@ typedef enum goldy_status {
 
 typedef enum goldy_dtype { GOLDY_BF16 = 0, GOLDY_F32 = 1 } goldy_dtype;
 
-/* One GEMM (Sec. 2.1.2).  Sizes and leading dimensions are in elements.
- * Supported now: trans_a = trans_b = 0, a = b = GOLDY_BF16, c = BF16 or F32,
- * M, N, K >= 0, lda >= K, ldb >= N, ldc >= N, lda and ldb multiples of 8
- * (16-byte rows for the tensor-memory-accelerator copies). */
+/* One GEMM (Sec. 2.1.2), or a strided batch of equal-sized GEMMs (the
+ * paper's B-GEMMs, Sec. 6.6): entry i computes C + i*stride_c = (A +
+ * i*stride_a)(B + i*stride_b).  Sizes, leading dimensions and strides are in
+ * elements.  Supported now: trans_a = trans_b = 0, a = b = GOLDY_BF16, c =
+ * BF16 or F32, M, N, K >= 0, lda >= K, ldb >= N, ldc >= N, lda and ldb
+ * multiples of 8 (16-byte rows for the tensor-memory-accelerator copies);
+ * batch >= 1 (1: a plain GEMM, strides ignored); for batch > 1 the entries
+ * do not overlap — stride_a >= M*lda, stride_b >= K*ldb, stride_c >= M*ldc —
+ * and stride_a, stride_b are multiples of 8. */
 typedef struct goldy_gemm_desc {
   int64_t M, N, K;
   int64_t lda, ldb, ldc;
   int32_t trans_a, trans_b;    /* the paper's T1, T2; only 0, 0 is supported */
   int32_t a_dtype, b_dtype, c_dtype;
   int32_t reserved;            /* must be 0 */
+  int64_t batch;               /* strided batch entries, >= 1 */
+  int64_t stride_a, stride_b, stride_c;
 } goldy_gemm_desc;
 
 typedef struct goldy_lut goldy_lut;
@@ -140,16 +147,21 @@ goldy_status goldy_variant_info_get(int id, goldy_variant_info* out);
 /* ---- lookup table (the dynamic logic's profiled data, Sec. 4.3) ---------
  * File format (little-endian): magic "GOLDYLUT", u32 version = 1, u32 entry
  * count, u32 variant-id bound, u32 SM count of the profiling GPU, 8 zero
- * bytes; then 16-byte entries {u8 lm, ln, lk, out_dtype; u8 pref_cd; u8 0;
+ * bytes; then 16-byte entries {u8 lm, ln, lk, out_dtype; u8 pref_cd; u8 flags;
  * u16 variant[5]} strictly sorted by (lm, ln, lk, out_dtype), where lm, ln,
  * lk are floor(log2) of M, N, K and variant[c] is the GO-Kernel for CD class
- * c in {1, 2, 4, 8, 16}.  GOLDY_ERR_LUT if the data is malformed or empty. */
+ * c in {1, 2, 4, 8, 16}; flags: how the bucket's GEMM runs with an
+ * element-wise op of its output size (see goldy_corun_plan) — bit 0: at once
+ * (else one after the other), bit 1: with the CD-2 GO-Kernel (else the CD-1
+ * kernel), bits 2-3: the op's grid-cap divisor 1, 2 or 4 as 0, 1, 2; other
+ * bits 0.  GOLDY_ERR_LUT if the data is malformed or empty. */
 goldy_status goldy_lut_load(const char* path, goldy_lut** out);
 goldy_status goldy_lut_from_memory(const void* data, size_t bytes, goldy_lut** out);
 void goldy_lut_free(goldy_lut* lut);
 
 /* Bucket key of one GEMM: (lm << 24) | (ln << 16) | (lk << 8) | c_dtype,
- * each log2 floored (0 for a size of 0) and clamped to 255. */
+ * each log2 floored (0 for a size of 0) and clamped to 255; a batched GEMM
+ * is bucketed by its rows over all entries (lm = floor log2(M * batch)). */
 goldy_status goldy_bucket_key(const goldy_gemm_desc* d, uint32_t* key);
 
 /* ---- planning (host only; makes no CUDA call) ---------------------------
@@ -164,10 +176,10 @@ goldy_status goldy_plan(const goldy_gemm_desc* descs, int n, const goldy_lut* lu
 /* ---- logistic-regression CD predictor (Sec. 4.3, Eq. 1) -----------------
  * The paper predicts each GEMM's preferred CD with a multi-class logistic
  * regression trained offline once per GPU.  Features (GOLDY_LR_FEATURES, in
- * this order): M, N, K, then for each CD class c in (1, 2, 4, 8, 16) three
- * numbers of the table's GO-Kernel for the GEMM's bucket at c: its CTAs of
- * work (output tiles x split-K slices; two CTAs per tile for a CTA-pair
- * kernel), its CTAs resident per SM, and its waves (CTAs of work over
+ * this order): M (times the batch), N, K, then for each CD class c in (1, 2,
+ * 4, 8, 16) three numbers of the table's GO-Kernel for the GEMM's bucket at
+ * c: its CTAs of work (output tiles of all batch entries x split-K slices;
+ * two CTAs per tile for a CTA-pair kernel), its CTAs resident per SM, and its waves (CTAs of work over
  * CTAs/SM x sm_count / grid-cap divisor, rounded up).  The model min-max
  * normalises them ((x - lo) / (hi - lo), 0 where hi == lo), scores each
  * class s_c = b_c + sum_j W[c][j] x_j (in j order, doubles, no fused
@@ -300,6 +312,56 @@ void goldy_exec_free(goldy_exec* e);
  * end event; *ms_per_rep = elapsed / reps.  Events live in the runs'
  * partition, so this also times work inside an SM partition. */
 goldy_status goldy_exec_time(const goldy_exec* const* execs, int n, int warmup, int reps, float* ms_per_rep);
+
+/* ---- a GEMM co-scheduled with a non-GEMM kernel (Sec. 8.1) --------------
+ * The paper co-runs a GEMM with an element-wise add of the GEMM's output size
+ * (2 kernels at once) and finds concurrency worth restricting for
+ * memory-bound GEMMs.  The non-GEMM here is Z = X + Y over n contiguous
+ * elements of `dtype` (bf16: each element widened to fp32, added in IEEE
+ * fp32 with round-to-nearest-even, rounded back to bf16 RNE; fp32: one IEEE
+ * fp32 addition), by a persistent grid-stride kernel whose grid is capped at
+ * 8 CTAs/SM x SMs / rc_div (rc_div 1, 2 or 4: GPU, GPU/2, GPU/4).
+ *
+ * Policies (goldy_corun_plan):
+ *   GOLDY_PLAN_SEQUENTIAL  isolation-tuned GEMM kernel, then the add, one stream
+ *   GOLDY_PLAN_DEFAULT     isolation-tuned GEMM kernel and the add (whole-GPU
+ *                          grid) at once on two streams
+ *   GOLDY_PLAN_GO          the table's CD-2 GO-Kernel and the add capped at
+ *                          GPU/2, at once
+ *   GOLDY_PLAN_AUTO        the configuration the table entry's flags record
+ *                          (profiled: the fastest of running at once with the
+ *                          CD-1 or CD-2 kernel and the op capped at GPU,
+ *                          GPU/2 or GPU/4, taken only when it beats one after
+ *                          the other by >= 5%), else SEQUENTIAL — concurrency
+ *                          restricted where it does not pay.
+ * The table's kernels are those of the GEMM's bucket (see goldy_lut_lookup). */
+typedef struct goldy_ewise_desc {
+  int64_t n;        /* elements (>= 0) */
+  int32_t dtype;    /* GOLDY_BF16 or GOLDY_F32, for X, Y and Z */
+  int32_t reserved; /* must be 0 */
+} goldy_ewise_desc;
+typedef struct goldy_corun goldy_corun;
+goldy_status goldy_corun_plan(const goldy_gemm_desc* gemm, const goldy_ewise_desc* ew, const goldy_lut* lut,
+                              int policy, goldy_corun** out);
+/* concurrent: 1 if the two kernels run at once (needs 2 streams); the GEMM's
+ * variant; the add's grid-cap divisor; device workspace bytes (split-K). */
+goldy_status goldy_corun_query(const goldy_corun* c, int* concurrent, int* gemm_variant, int* add_rc_div,
+                               size_t* workspace_bytes);
+/* Enqueue: the GEMM C = A B on streams[0]; the add on streams[1] (forked
+ * from and joined back into streams[0]) when concurrent, else on streams[0]
+ * after the GEMM.  X, Y, Z: device arrays of n elements; the vector path
+ * needs them 16-byte aligned (others take a scalar path).  Asynchronous. */
+goldy_status goldy_corun_run(const goldy_corun* c, const void* A, const void* B, void* C, void* workspace,
+                             size_t workspace_bytes, const void* X, const void* Y, void* Z, void* const* streams,
+                             int n_streams);
+/* The same, recorded once as a prepared run (see goldy_exec_create). */
+goldy_status goldy_corun_exec_create(const goldy_corun* c, const void* A, const void* B, void* C, void* workspace,
+                                     size_t workspace_bytes, const void* X, const void* Y, void* Z,
+                                     void* const* streams, int n_streams, goldy_exec** out);
+void goldy_corun_free(goldy_corun* c);
+
+/* The element-wise add alone on one stream (rc_div 1, 2 or 4). */
+goldy_status goldy_ewise_add(const void* X, const void* Y, void* Z, int64_t n, int dtype, int rc_div, void* stream);
 
 /* ---- SM partitions (the paper's CU-partition study, Sec. 6.7) -----------
  * A partition is a CUDA green context owning a subset of the GPU's SMs plus

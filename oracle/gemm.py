@@ -165,3 +165,17 @@ __all__ = ["gemm", "gemm_rows", "gemm_entries", "gemm_python", "bf16_decode",
 
 if os.environ.get("GOLDY_ORACLE_THREADS"):
     set_threads(int(os.environ["GOLDY_ORACLE_THREADS"]))
+
+
+def gemm_batched(a_bits: np.ndarray, b_bits: np.ndarray) -> np.ndarray:
+    """A strided batch of GEMMs (Sec. 6.6's B-GEMMs): entry i of the result
+    is gemm(a_bits[i], b_bits[i]) for a_bits (batch x M x K) and b_bits
+    (batch x K x N)."""
+    a_bits = _as_bits(a_bits)
+    b_bits = _as_bits(b_bits)
+    if a_bits.ndim != 3 or b_bits.ndim != 3 or a_bits.shape[0] != b_bits.shape[0]:
+        raise ValueError("batched operands must be (batch, rows, cols) with equal batch")
+    out = np.empty((a_bits.shape[0], a_bits.shape[1], b_bits.shape[2]), dtype=np.float64)
+    for i in range(a_bits.shape[0]):
+        out[i] = gemm(a_bits[i], b_bits[i])
+    return out

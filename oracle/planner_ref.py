@@ -9,7 +9,8 @@ Python and independently of the product's C++ planner, how a schedule follows
 from the table:
 
 1. Bucket each GEMM by its sizes: key = (floor(log2 M), floor(log2 N),
-   floor(log2 K), output dtype).  The paper's predictor reads M, N and K among
+   floor(log2 K), output dtype); a strided batch of GEMMs counts its rows
+   over all entries (M * batch).  The paper's predictor reads M, N and K among
    its features (Sec. 4.3); a log2 bucket is this table's stand-in for them.
 2. Look the key up.  A key the table lacks takes the stored key nearest in
    L1 distance over the three log2 sizes, a differing output dtype adding 16;
@@ -41,7 +42,9 @@ Binary formats written out here, independently of the C++ code:
 LUT file (little-endian): 8-byte magic ``GOLDYLUT``, u32 version (1), u32
 entry count, u32 variant-id bound, u32 SM count, 8 reserved bytes; then
 16-byte entries ``u8 lm, u8 ln, u8 lk, u8 out_dtype, u8 pref_cd, u8 flags,
-u16 variant[5]`` sorted strictly by (lm, ln, lk, out_dtype).
+u16 variant[5]`` sorted strictly by (lm, ln, lk, out_dtype); flags record how
+the bucket's GEMM runs with an element-wise op (bit 0 at once, bit 1 the CD-2
+kernel, bits 2-3 the op's grid-cap divisor 1/2/4 as 0/1/2), other bits 0.
 
 Schedule bytes (little-endian u32 words): ``GSCH`` magic, version (1),
 n_gemms, n_groups, max_streams, flags; per group: cd, size, members...; per
@@ -83,6 +86,7 @@ class Entry:
     key: Tuple[int, int, int, int]
     pref_cd: int
     variants: Tuple[int, int, int, int, int]
+    flags: int = 0          # co-run with an element-wise op: bit 0 at once, bit 1 CD-2 kernel, bits 2-3 op cap
 
 
 def parse_lut(data: bytes) -> Tuple[List[Entry], int]:
@@ -98,7 +102,7 @@ def parse_lut(data: bytes) -> Tuple[List[Entry], int]:
     entries: List[Entry] = []
     prev = None
     for e in range(n):
-        lm, ln, lk, out, pref, _flags = struct.unpack_from("<6B", data, 32 + 16 * e)
+        lm, ln, lk, out, pref, flags = struct.unpack_from("<6B", data, 32 + 16 * e)
         vs = struct.unpack_from("<5H", data, 32 + 16 * e + 6)
         key = (lm, ln, lk, out)
         if prev is not None and key <= prev:
@@ -107,10 +111,12 @@ def parse_lut(data: bytes) -> Tuple[List[Entry], int]:
             raise LutError("bad dtype")
         if pref not in CD_CLASSES:
             raise LutError("bad preferred cd")
+        if flags & ~0x0F or (flags >> 2) & 3 == 3:
+            raise LutError("unknown flag bits")
         if any(v >= n_variants for v in vs):
             raise LutError("variant out of range")
         prev = key
-        entries.append(Entry(key, pref, tuple(vs)))
+        entries.append(Entry(key, pref, tuple(vs), flags))
     if not entries:
         raise LutError("empty table")
     return entries, n_variants
@@ -120,7 +126,7 @@ def write_lut(entries: Sequence[Entry], n_variants: int, sm_count: int = 0) -> b
     out = bytearray(LUT_MAGIC)
     out += struct.pack("<IIIIII", 1, len(entries), n_variants, sm_count, 0, 0)
     for e in sorted(entries, key=lambda x: x.key):
-        out += struct.pack("<6B", *e.key, e.pref_cd, 0)
+        out += struct.pack("<6B", *e.key, e.pref_cd, e.flags)
         out += struct.pack("<5H", *e.variants)
     return bytes(out)
 
@@ -160,6 +166,7 @@ class Desc:
     N: int
     K: int
     out_dtype: int
+    batch: int = 1          # strided batch entries (Sec. 6.6's B-GEMMs); bucketed by M * batch rows
 
 
 def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
@@ -173,7 +180,7 @@ def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
     forced = (flags >> 8) & 0xFF
     if (flags & ~0xFF1F) or policy > POLICY_FORCE_CD or (policy == POLICY_FORCE_CD and forced < 1):
         raise PlanError("bad flags")
-    keys = [bucket_key(d.M, d.N, d.K, d.out_dtype) for d in descs]
+    keys = [bucket_key(d.M * d.batch, d.N, d.K, d.out_dtype) for d in descs]
     ents = [lookup(entries, k) for k in keys]
 
     def one_group(cd: int, cls_cd: Optional[int]):
@@ -194,7 +201,7 @@ def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
         blocks = []
         for k in sorted(set(keys)):
             members = [i for i in range(n) if keys[i] == k]
-            flops = sum(2 * descs[i].M * descs[i].N * descs[i].K for i in members)
+            flops = sum(2 * descs[i].M * descs[i].N * descs[i].K * descs[i].batch for i in members)
             blocks.append((-flops, k, members, ents[members[0]].pref_cd))
         blocks.sort(key=lambda b: (b[0], b[1]))
         merged = []                         # each: (members, min pref, n keys)
@@ -243,3 +250,28 @@ def preferred_cd(speedup: dict, gain: float = 0.05, near: float = 0.01) -> int:
     if best < 1.0 + gain:
         return 1
     return min(cd for cd, s in cands.items() if s >= best * (1.0 - near))
+
+
+def corun_plan(d: Desc, lut_bytes: bytes, policy: int) -> Tuple[int, int, int]:
+    """A GEMM co-scheduled with an element-wise op over its output (Sec. 8.1):
+    (concurrent, GEMM variant, grid-cap divisor of the element-wise kernel).
+    sequential: isolation-tuned kernel, then the op; default: the
+    isolation-tuned kernel and the op (whole GPU) at once; go: the CD-2
+    GO-Kernel and the op capped at half the GPU, at once; automatic: the
+    configuration the table entry's flags record (bit 0 at once, bit 1 the
+    CD-2 kernel instead of the CD-1 one, bits 2-3 the op's cap 1, 2 or 4),
+    one after the other when bit 0 is clear — concurrency restricted where it
+    does not help."""
+    entries, _ = parse_lut(lut_bytes)
+    if policy not in (POLICY_AUTO, POLICY_SEQUENTIAL, POLICY_DEFAULT, POLICY_GO):
+        raise PlanError("bad policy")
+    e = lookup(entries, bucket_key(d.M * d.batch, d.N, d.K, d.out_dtype))
+    if policy == POLICY_SEQUENTIAL:
+        return 0, e.variants[0], 1
+    if policy == POLICY_DEFAULT:
+        return 1, e.variants[0], 1
+    if policy == POLICY_GO:
+        return 1, e.variants[1], 2
+    if e.flags & 1:
+        return 1, e.variants[1] if e.flags & 2 else e.variants[0], 1 << ((e.flags >> 2) & 3)
+    return 0, e.variants[0], 1

@@ -6,7 +6,7 @@ GEMM to its preferred concurrency degree (Sec. 4.3, Eq. 1).  This module
 restates, in plain Python and independently of the product's C++ planner,
 what the trained model computes at planning time:
 
-1. Features (Sec. 4.3): the GEMM's M, N and K, and for each CD class c in
+1. Features (Sec. 4.3): the GEMM's M (times its batch), N and K, and for each CD class c in
    (1, 2, 4, 8, 16) three numbers of the GO-Kernel the table assigns to the
    GEMM's bucket at that CD — its work-group count (here: CTAs of work, i.e.
    output tiles x split-K slices, two CTAs per tile for a CTA-pair kernel),
@@ -112,15 +112,16 @@ def write_model(m: Model) -> bytes:
     return bytes(out)
 
 
-def kernel_features(M: int, N: int, variant: int, sm_count: int) -> Tuple[int, int, int]:
-    """(CTAs of work, CTAs per SM, waves) of one GO-Kernel on an M x N output."""
+def kernel_features(M: int, N: int, variant: int, sm_count: int, batch: int = 1) -> Tuple[int, int, int]:
+    """(CTAs of work, CTAs per SM, waves) of one GO-Kernel on `batch` M x N
+    outputs."""
     kind = variant // 12
     split = SPLITS[(variant // 3) % 4]
     rc_div = RC_DIVS[variant % 3]
     rows, cols, per_sm, per_tile = KIND_GEOMETRY[kind]
     if per_tile > 1:
         split = 1
-    tiles = -(-M // rows) * -(-N // cols)
+    tiles = batch * (-(-M // rows)) * (-(-N // cols))
     ctas = tiles * split * per_tile
     cap = max(per_tile, per_sm * sm_count // rc_div)
     waves = -(-ctas // cap)
@@ -128,9 +129,9 @@ def kernel_features(M: int, N: int, variant: int, sm_count: int) -> Tuple[int, i
 
 
 def features(d: pr.Desc, entry: pr.Entry, sm_count: int) -> List[float]:
-    x = [float(d.M), float(d.N), float(d.K)]
+    x = [float(d.M * d.batch), float(d.N), float(d.K)]
     for v in entry.variants:
-        x += [float(f) for f in kernel_features(d.M, d.N, v, sm_count)]
+        x += [float(f) for f in kernel_features(d.M, d.N, v, sm_count, d.batch)]
     return x
 
 
@@ -165,7 +166,7 @@ def predict_class(s: Sequence[float]) -> int:
 
 
 def predict_cd(d: pr.Desc, entries: Sequence[pr.Entry], m: Model) -> int:
-    e = pr.lookup(entries, pr.bucket_key(d.M, d.N, d.K, d.out_dtype))
+    e = pr.lookup(entries, pr.bucket_key(d.M * d.batch, d.N, d.K, d.out_dtype))
     s = scores(normalise(features(d, e, m.sm_count), m), m)
     return pr.CD_CLASSES[predict_class(s)]
 
@@ -180,7 +181,7 @@ def plan(descs: Sequence[pr.Desc], lut_bytes: bytes, model_bytes: Optional[bytes
     entries, _ = pr.parse_lut(lut_bytes)
     prefs = {}
     for d in descs:
-        k = pr.bucket_key(d.M, d.N, d.K, d.out_dtype)
+        k = pr.bucket_key(d.M * d.batch, d.N, d.K, d.out_dtype)
         prefs[k] = min(prefs.get(k, pr.CD_CLASSES[-1]), predict_cd(d, entries, m))
     return _plan_with_prefs(descs, entries, prefs, flags)
 
@@ -191,12 +192,12 @@ def _plan_with_prefs(descs, entries, prefs, flags):
         raise pr.PlanError("bad count")
     if flags & ~0xFF1F:
         raise pr.PlanError("bad flags")
-    keys = [pr.bucket_key(d.M, d.N, d.K, d.out_dtype) for d in descs]
+    keys = [pr.bucket_key(d.M * d.batch, d.N, d.K, d.out_dtype) for d in descs]
     ents = [pr.lookup(entries, k) for k in keys]
     blocks = []
     for k in sorted(set(keys)):
         members = [i for i in range(n) if keys[i] == k]
-        flops = sum(2 * descs[i].M * descs[i].N * descs[i].K for i in members)
+        flops = sum(2 * descs[i].M * descs[i].N * descs[i].K * descs[i].batch for i in members)
         blocks.append((-flops, k, members, prefs[k]))
     blocks.sort(key=lambda b: (b[0], b[1]))
     merged = []

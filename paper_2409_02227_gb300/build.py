@@ -52,6 +52,7 @@ def _jobs(ptxas_verbose: bool):
                              "-c", os.path.join(CSRC, "planner.cpp")]))
     jobs.append(("runtime", cu + ["-c", os.path.join(CSRC, "runtime.cu")]))
     jobs.append(("noalloc", cu + ["-c", os.path.join(CSRC, "noalloc.cu")]))
+    jobs.append(("ewise", cu + ["-c", os.path.join(CSRC, "ewise.cu")]))
     for k in range(NUM_KINDS):
         jobs.append((f"kernels_k{k}", cu + [f"-DGOLDY_KIND={k}", "-c", os.path.join(CSRC, "kernels.cu")]))
     return jobs

@@ -2,7 +2,9 @@
 //
 // What it computes (Sec. 2.1.2): C = A * B for A (M x K, row-major), B
 // (K x N, row-major), fp32 accumulation, fp32 or bf16 (round-to-nearest-even)
-// output.  Several GEMMs may share one launch (the launch's "units" are the
+// output; a strided-batched GEMM (Sec. 6.6's B-GEMMs) is `batch` such
+// products at fixed strides, its tiles numbered batch entry by batch entry.
+// Several GEMMs may share one launch (the launch's "units" are the
 // concatenation of their tiles).
 //
 // How (Sec. 2.1.3's tiled GEMM re-expressed for tcgen05):
@@ -47,20 +49,38 @@ struct GemmWork {
   float* ws_part;       // split-K partial tiles (null when split == 1)
   uint32_t* ws_cnt;     // split-K arrival counter per tile
   int64_t ldc;
+  int64_t c_bstride;    // elements between the C matrices of consecutive batch entries
   int32_t m, n, k;
-  int32_t tiles_m, tiles_n;
+  int32_t tiles_m, tiles_n;   // tiles of one batch entry
   int32_t split;        // K-range split, 1 <= split <= k_blocks
   int32_t k_blocks;     // ceil(K / 64)
   int32_t unit_begin;   // first unit of this GEMM within the launch
   int32_t c_tma;        // 1: C is written through tmap_c by TMA stores
-  int32_t pad_[2];
+  int32_t batch;        // strided batch entries (1: a plain GEMM)
 };
+
+// Where one batch entry's C lives: the store helpers' view of a GemmWork.
+struct CView {
+  void* c;
+  int64_t ldc;
+  int32_t m, n;
+};
+
+template <bool OUT_BF16>
+__device__ __forceinline__ CView c_view(const GemmWork& w, int b) {
+  CView v;
+  v.c = static_cast<char*>(w.c) + int64_t(b) * w.c_bstride * (OUT_BF16 ? 2 : 4);
+  v.ldc = w.ldc;
+  v.m = w.m;
+  v.n = w.n;
+  return v;
+}
 
 template <int MAXG>
 struct LaunchParams {
-  CUtensorMap tmap_a[MAXG];   // A: dims {K, M}, box {64, rows of the A tile}
-  CUtensorMap tmap_b[MAXG];   // B: dims {N, K}, box {64, 64}
-  CUtensorMap tmap_c[MAXG];   // C: dims {N, M}, box {128-byte row, 128 rows} (when g[].c_tma)
+  CUtensorMap tmap_a[MAXG];   // A: dims {K, M, batch}, box {64, rows of the A tile, 1}
+  CUtensorMap tmap_b[MAXG];   // B: dims {N, K, batch}, box {64, 64, 1}
+  CUtensorMap tmap_c[MAXG];   // C: dims {N, M, batch}, box {128-byte row, 128 rows, 1} (when g[].c_tma)
   GemmWork g[MAXG];
   int32_t n_gemms;
   int32_t total_units;
@@ -95,7 +115,7 @@ enum : int {
 };
 
 struct UnitCoord {
-  int g, tile, s, tm, tn, kb0, kb1;
+  int g, tile, s, b, tm, tn, kb0, kb1;   // tile counts over all batch entries; b = batch entry
 };
 
 template <int MAXG>
@@ -109,8 +129,11 @@ __device__ __forceinline__ UnitCoord decode_unit(const LaunchParams<MAXG>& p, in
   c.g = g;
   c.tile = local / w.split;
   c.s = local - c.tile * w.split;
-  c.tm = c.tile % w.tiles_m;
-  c.tn = c.tile / w.tiles_m;
+  const int per_batch = w.tiles_m * w.tiles_n;
+  c.b = c.tile / per_batch;
+  const int t = c.tile - c.b * per_batch;
+  c.tm = t % w.tiles_m;
+  c.tn = t / w.tiles_m;
   c.kb0 = (c.s * w.k_blocks) / w.split;
   c.kb1 = ((c.s + 1) * w.k_blocks) / w.split;
   return c;
@@ -129,7 +152,7 @@ __device__ __forceinline__ void raise_error(int* err, volatile int* abort_flag, 
 //  !SWAP: row `r` of the tile is C row m0 + r; columns n0 + c0 .. +31.
 //   SWAP: row `r` of the tile is C column n0 + r; columns are C rows m0 + c0 .. +31.
 template <bool SWAP, bool OUT_BF16>
-__device__ __forceinline__ void store_chunk(const GemmWork& w, int m0, int n0, int r, int c0, const float (&v)[32]) {
+__device__ __forceinline__ void store_chunk(const CView& w, int m0, int n0, int r, int c0, const float (&v)[32]) {
   if (!SWAP) {
     const int64_t row = int64_t(m0) + r;
     if (row >= w.m) return;
@@ -186,7 +209,7 @@ __device__ __forceinline__ void store_chunk(const GemmWork& w, int m0, int n0, i
 // Store 4 consecutive accumulator columns (acc_col .. acc_col+3) of
 // accumulator row acc_row, mapped to C as in store_chunk.
 template <bool SWAP, bool OUT_BF16>
-__device__ __forceinline__ void store_quad(const GemmWork& w, int m0, int n0, int acc_row, int acc_col, float4 a) {
+__device__ __forceinline__ void store_quad(const CView& w, int m0, int n0, int acc_row, int acc_col, float4 a) {
   const float v[4] = {a.x, a.y, a.z, a.w};
   if (!SWAP) {
     const int64_t row = int64_t(m0) + acc_row;
@@ -237,7 +260,7 @@ __device__ __forceinline__ void store_quad(const GemmWork& w, int m0, int n0, in
 // 0, 1, ..., S-1, and stores them.  Partial layout: [chunk][float4][row].
 // Per batch, IB items x S partials are loaded before any is added.
 template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
-__device__ __forceinline__ void reduce_slice(const GemmWork& w, const float4* tile_parts, int rank, int m0, int n0,
+__device__ __forceinline__ void reduce_slice(const CView& w, const float4* tile_parts, int rank, int m0, int n0,
                                              int t) {
   constexpr int R = 128 / S;
   constexpr int COLS4 = MMA_N / 4;
@@ -281,7 +304,7 @@ __device__ __forceinline__ void reduce_slice(const GemmWork& w, const float4* ti
 // clips rows and columns outside C.
 template <int MMA_N, bool OUT_BF16>
 __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t staging, uint32_t& stg, uint32_t taddr,
-                                               int r, int et, int m0, int n0) {
+                                               int r, int et, int m0, int n0, int b) {
   constexpr int CHUNK = OUT_BF16 ? 64 : 32;
 #pragma unroll 1
   for (int c0 = 0; c0 < MMA_N; c0 += CHUNK) {
@@ -324,7 +347,7 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
     ptx::fence_proxy_async_smem();
     ptx::named_bar_sync(1, 128);
     if (et == 0) {
-      ptx::tma_store_2d(tmap_c, buf, n0 + c0, m0);
+      ptx::tma_store_3d(tmap_c, buf, n0 + c0, m0, b);
       ptx::bulk_commit_group();
     }
     ++stg;
@@ -335,7 +358,7 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
 // but partial s is read from the shared memory of cluster CTA s (same
 // [chunk][float4][row] layout at `part_smem` in every CTA).
 template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
-__device__ __forceinline__ void reduce_slice_dsmem(const GemmWork& w, uint32_t part_smem, int rank, int m0, int n0,
+__device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part_smem, int rank, int m0, int n0,
                                                    int t) {
   constexpr int R = 128 / S;
   constexpr int COLS4 = MMA_N / 4;
@@ -486,13 +509,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           const uint32_t ys = xs + X_BYTES;
           const int k0 = kb * 64;
           if (!SWAP) {
-            ptx::tma_load_2d(xs, ta, fb, k0, m0);
+            ptx::tma_load_3d(xs, ta, fb, k0, m0, c.b);
 #pragma unroll
-            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_2d(ys + j * 8192, tb, fb, n0 + 64 * j, k0);
+            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_3d(ys + j * 8192, tb, fb, n0 + 64 * j, k0, c.b);
           } else {
 #pragma unroll
-            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_2d(xs + j * 8192, tb, fb, n0 + 64 * j, k0);
-            ptx::tma_load_2d(ys, ta, fb, k0, m0);
+            for (int j = 0; j < B_BOXES; ++j) ptx::tma_load_3d(xs + j * 8192, tb, fb, n0 + 64 * j, k0, c.b);
+            ptx::tma_load_3d(ys, ta, fb, k0, m0, c.b);
           }
           if (issued == 0) trace_stamp(trace, kTrFirstLoad);
           issued |= 1u << stage;
@@ -591,11 +614,12 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const bool first_unit = (u == int(blockIdx.x));
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
       const GemmWork& w = p.g[c.g];
+      const CView cv = c_view<OUT_BF16>(w, c.b);
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);
       if (EPI_TMA && w.split == 1 && w.c_tma) {
-        store_tile_tma<MMA_N, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0);
+        store_tile_tma<MMA_N, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
       } else if (w.split == 1) {
 #pragma unroll 1
         for (int c0 = 0; c0 < MMA_N; c0 += 32) {
@@ -606,7 +630,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
-          store_chunk<SWAP, OUT_BF16>(w, m0, n0, r, c0, v);
+          store_chunk<SWAP, OUT_BF16>(cv, m0, n0, r, c0, v);
         }
       } else if (kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x)) {
         // ---- cluster split-K on chip: one unit per CTA, so the ring's shared
@@ -646,9 +670,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         }
         if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
         switch (w.split) {
-          case 2: reduce_slice_dsmem<MMA_N, 2, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
-          case 4: reduce_slice_dsmem<MMA_N, 4, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
-          case 8: reduce_slice_dsmem<MMA_N, 8, SWAP, OUT_BF16>(w, part_smem, c.s, m0, n0, et); break;
+          case 2: reduce_slice_dsmem<MMA_N, 2, SWAP, OUT_BF16>(cv, part_smem, c.s, m0, n0, et); break;
+          case 4: reduce_slice_dsmem<MMA_N, 4, SWAP, OUT_BF16>(cv, part_smem, c.s, m0, n0, et); break;
+          case 8: reduce_slice_dsmem<MMA_N, 8, SWAP, OUT_BF16>(cv, part_smem, c.s, m0, n0, et); break;
           default: break;
         }
       } else {
@@ -692,9 +716,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
           const float4* tile_parts = part_base + size_t(c.tile * w.split) * TILE_F4;
           switch (w.split) {
-            case 2: reduce_slice<MMA_N, 2, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
-            case 4: reduce_slice<MMA_N, 4, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
-            case 8: reduce_slice<MMA_N, 8, SWAP, OUT_BF16>(w, tile_parts, c.s, m0, n0, et); break;
+            case 2: reduce_slice<MMA_N, 2, SWAP, OUT_BF16>(cv, tile_parts, c.s, m0, n0, et); break;
+            case 4: reduce_slice<MMA_N, 4, SWAP, OUT_BF16>(cv, tile_parts, c.s, m0, n0, et); break;
+            case 8: reduce_slice<MMA_N, 8, SWAP, OUT_BF16>(cv, tile_parts, c.s, m0, n0, et); break;
             default: break;
           }
         } else {
@@ -750,7 +774,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
                 }
               }
             }
-            store_chunk<SWAP, OUT_BF16>(w, m0, n0, r, c0, v);
+            store_chunk<SWAP, OUT_BF16>(cv, m0, n0, r, c0, v);
           }
           if (et == 0) w.ws_cnt[c.tile] = 0u;     // leave the counter zeroed for the next run
         }

@@ -119,9 +119,9 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
           const uint32_t xs = tiles_base + stage * STAGE_BYTES;
           const uint32_t ys = xs + A_BYTES;
           const int k0 = kb * 64;
-          ptx::tma_load_2d_pair(xs, ta, fb, k0, m0);
-          ptx::tma_load_2d_pair(ys, tb, fb, n0, k0);
-          ptx::tma_load_2d_pair(ys + 8192, tb, fb, n0 + 64, k0);
+          ptx::tma_load_3d_pair(xs, ta, fb, k0, m0, c.b);
+          ptx::tma_load_3d_pair(ys, tb, fb, n0, k0, c.b);
+          ptx::tma_load_3d_pair(ys + 8192, tb, fb, n0 + 64, k0, c.b);
           if (issued == 0) trace_stamp(trace, kTrFirstLoad);
           issued |= 1u << stage;
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
@@ -223,11 +223,12 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       const bool first_unit = (u == pair);
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
       const GemmWork& w = p.g[c.g];
+      const CView cv = c_view<OUT_BF16>(w, c.b);
       const int m0 = c.tm * 256 + int(rank) * 128;
       const int n0 = c.tn * 256;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
       if (w.c_tma) {
-        store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0);
+        store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
       } else {
 #pragma unroll 1
         for (int c0 = 0; c0 < 256; c0 += 32) {
@@ -238,7 +239,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
-          store_chunk<false, OUT_BF16>(w, m0, n0, r, c0, v);
+          store_chunk<false, OUT_BF16>(cv, m0, n0, r, c0, v);
         }
       }
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstStore);

@@ -136,6 +136,19 @@ const void* kernel_fn_k8(int out_bf16, int fused);
 const void* kernel_fn_k9(int out_bf16, int fused);
 const void* kernel_fn_k10(int out_bf16, int fused);
 
+// Element-wise add (ewise.cu): Z = X + Y over n elements.
+struct EwiseParams {
+  const void* x;
+  const void* y;
+  void* z;
+  int64_t n;
+  int32_t vec_ok;   // all three pointers 16-byte aligned
+  int32_t pad;
+};
+constexpr int kEwiseThreads = 256;
+constexpr int kEwiseCtasPerSm = 8;
+const void* ewise_kernel_fn(int bf16);
+
 }  // namespace goldy
 
 struct goldy_schedule {
@@ -145,6 +158,17 @@ struct goldy_schedule {
   std::vector<goldy::GemmPlan> gemms;
   std::vector<goldy::Group> groups;
   goldy::Runtime* rt = nullptr;   // created on first goldy_run
+};
+
+// A GEMM co-scheduled with an element-wise add (planner.cpp builds it,
+// runtime.cu runs it).
+struct goldy_corun {
+  goldy_schedule* gemm = nullptr;   // one GEMM with the chosen variant (owned)
+  goldy_ewise_desc ew{};
+  int policy = 0;
+  int concurrent = 0;
+  int add_rc_div = 1;
+  goldy::Runtime* rt = nullptr;     // fork/join events, created on first run
 };
 
 namespace goldy {

@@ -81,6 +81,7 @@ extern "C" goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int vari
   goldy_status st = check_desc(*desc, 0);
   if (st != GOLDY_OK) return st;
   if (variant < 0 || variant >= kNumVariants) return fail(GOLDY_ERR_INVALID_ARG, "variant id out of range");
+  if (desc->batch != 1) return fail(GOLDY_ERR_UNSUPPORTED, "batched GEMMs go through goldy_run");
 
   GemmPlan gp;
   gp.desc = *desc;

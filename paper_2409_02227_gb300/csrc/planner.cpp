@@ -65,6 +65,15 @@ goldy_status check_desc(const goldy_gemm_desc& d, int i) {
     return fail(GOLDY_ERR_INVALID_ARG, at + "lda and ldb must be multiples of 8 (16-byte rows)");
   if (d.lda >= (int64_t(1) << 36) || d.ldb >= (int64_t(1) << 36))
     return fail(GOLDY_ERR_INVALID_ARG, at + "leading dimension too large");
+  if (d.batch < 1 || d.batch >= lim) return fail(GOLDY_ERR_INVALID_ARG, at + "batch must be in 1 .. 2^31-1");
+  if (d.batch > 1) {
+    if (d.stride_a < d.M * d.lda || d.stride_b < d.K * d.ldb || d.stride_c < d.M * d.ldc)
+      return fail(GOLDY_ERR_INVALID_ARG, at + "batch entries overlap (stride smaller than one entry)");
+    if (d.stride_a % 8 != 0 || d.stride_b % 8 != 0)
+      return fail(GOLDY_ERR_INVALID_ARG, at + "stride_a and stride_b must be multiples of 8 (16 bytes)");
+    if (d.stride_a >= (int64_t(1) << 36) || d.stride_b >= (int64_t(1) << 36) || d.stride_c >= (int64_t(1) << 36))
+      return fail(GOLDY_ERR_INVALID_ARG, at + "batch stride too large");
+  }
   return GOLDY_OK;
 }
 
@@ -89,6 +98,7 @@ namespace {
 struct LutEntry {
   uint8_t lm, ln, lk, out;
   uint8_t pref_cd;
+  uint8_t flags;   // co-run with an element-wise op: bit 0 at once, bit 1 CD-2 kernel, bits 2-3 add cap
   uint16_t variant[5];
   uint32_t key() const { return (uint32_t(lm) << 24) | (uint32_t(ln) << 16) | (uint32_t(lk) << 8) | out; }
 };
@@ -134,8 +144,9 @@ extern "C" goldy_status goldy_lut_from_memory(const void* data, size_t bytes, go
     x.lk = q[2];
     x.out = q[3];
     x.pref_cd = q[4];
+    x.flags = q[5];
     for (int c = 0; c < 5; ++c) x.variant[c] = rd16(q + 6 + 2 * c);
-    bool bad = (x.out != GOLDY_BF16 && x.out != GOLDY_F32);
+    bool bad = (x.out != GOLDY_BF16 && x.out != GOLDY_F32) || (x.flags & ~0x0Fu) != 0 || ((x.flags >> 2) & 3u) == 3u;
     bool pref_ok = false;
     for (int c : kCdClasses) pref_ok |= (x.pref_cd == c);
     bad |= !pref_ok;
@@ -226,7 +237,8 @@ extern "C" goldy_status goldy_predictor_load(const char* path, goldy_predictor**
 extern "C" void goldy_predictor_free(goldy_predictor* m) { delete m; }
 
 static uint32_t bucket_key(const goldy_gemm_desc& d) {
-  return (uint32_t(floor_log2_u8(d.M)) << 24) | (uint32_t(floor_log2_u8(d.N)) << 16) |
+  return (uint32_t(floor_log2_u8(d.M * std::max<int64_t>(d.batch, 1))) << 24) |
+         (uint32_t(floor_log2_u8(d.N)) << 16) |
          (uint32_t(floor_log2_u8(d.K)) << 8) | uint32_t(d.c_dtype & 0xFF);
 }
 
@@ -261,13 +273,14 @@ extern "C" goldy_status goldy_lut_lookup(const goldy_lut* lut, const goldy_gemm_
   return ok();
 }
 
-// Features of one GEMM for the predictor (Sec. 4.3): M, N, K, then for each
-// CD class the table's GO-Kernel's CTAs of work (tiles x split-K slices, two
-// CTAs per tile for a CTA pair), CTAs resident per SM, and waves (CTAs of work
-// over the capped persistent grid, rounded up).
+// Features of one GEMM for the predictor (Sec. 4.3): M (times the batch), N,
+// K, then for each CD class the table's GO-Kernel's CTAs of work (tiles over
+// all batch entries x split-K slices, two CTAs per tile for a CTA pair), CTAs
+// resident per SM, and waves (CTAs of work over the capped persistent grid,
+// rounded up).
 static void lr_features(const goldy_gemm_desc& d, const LutEntry& e, int64_t sm_count,
                         double x[GOLDY_LR_FEATURES]) {
-  x[0] = double(d.M);
+  x[0] = double(d.M * d.batch);
   x[1] = double(d.N);
   x[2] = double(d.K);
   for (int c = 0; c < 5; ++c) {
@@ -275,7 +288,7 @@ static void lr_features(const goldy_gemm_desc& d, const LutEntry& e, int64_t sm_
     const KindInfo& k = kKinds[v.kind];
     const int64_t per_tile = k.pair ? 2 : 1;
     const int64_t split = k.pair ? 1 : v.split;
-    const int64_t ctas = ceil_div(d.M, tile_rows(k)) * ceil_div(d.N, tile_cols(k)) * split * per_tile;
+    const int64_t ctas = d.batch * ceil_div(d.M, tile_rows(k)) * ceil_div(d.N, tile_cols(k)) * split * per_tile;
     const int64_t cap = std::max<int64_t>(per_tile, int64_t(k.ctas_per_sm) * sm_count / v.rc_div);
     x[3 + 3 * c] = double(ctas);
     x[4 + 3 * c] = double(k.ctas_per_sm);
@@ -347,7 +360,7 @@ void finalize_schedule(goldy_schedule* s) {
     gp.tiles_n = ceil_div(gp.desc.N, tile_cols(k));
     gp.k_blocks = ceil_div(gp.desc.K, kBlockK);
     gp.split = k.pair ? 1 : int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
-    const int64_t tiles = gp.tiles_m * gp.tiles_n;
+    const int64_t tiles = gp.tiles_m * gp.tiles_n * gp.desc.batch;   // over all batch entries
     gp.units = (gp.desc.K > 0) ? tiles * gp.split : 0;
     gp.ws_part_off = gp.ws_cnt_off = gp.ws_bytes = 0;
     if (gp.split > 1 && tiles > 0) {
@@ -440,8 +453,8 @@ extern "C" goldy_status goldy_plan_ex(const goldy_gemm_desc* descs, int n, const
       std::vector<Block> blocks;
       for (int i = 0; i < n; ++i) {
         auto it = std::find_if(blocks.begin(), blocks.end(), [&](const Block& b) { return b.key == keys[i]; });
-        const unsigned __int128 f =
-            (unsigned __int128)2 * uint64_t(descs[i].M) * uint64_t(descs[i].N) * uint64_t(descs[i].K);
+        const unsigned __int128 f = (unsigned __int128)2 * uint64_t(descs[i].M) * uint64_t(descs[i].N) *
+                                    uint64_t(descs[i].K) * uint64_t(descs[i].batch);
         if (it == blocks.end()) {
           blocks.push_back({keys[i], f, {i}, pref[i]});
         } else {
@@ -618,4 +631,72 @@ extern "C" goldy_status goldy_variant_info_get(int id, goldy_variant_info* out) 
   out->cta_pair = k.pair ? 2 : 1;
   std::snprintf(out->name, sizeof(out->name), "%s_s%d_rc%d", k.name, v.split, v.rc_div);
   return ok();
+}
+
+// ---------------------------------------------------------------------------
+// A GEMM co-scheduled with an element-wise add (Sec. 8.1)
+// ---------------------------------------------------------------------------
+extern "C" goldy_status goldy_corun_plan(const goldy_gemm_desc* gemm, const goldy_ewise_desc* ew,
+                                         const goldy_lut* lut, int policy, goldy_corun** out) {
+  if (!gemm || !ew || !out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  if (!lut) return fail(GOLDY_ERR_LUT, "no lookup table");
+  if (policy != GOLDY_PLAN_AUTO && policy != GOLDY_PLAN_SEQUENTIAL && policy != GOLDY_PLAN_DEFAULT &&
+      policy != GOLDY_PLAN_GO)
+    return fail(GOLDY_ERR_INVALID_ARG, "bad policy");
+  if (ew->n < 0 || ew->reserved != 0 || (ew->dtype != GOLDY_BF16 && ew->dtype != GOLDY_F32))
+    return fail(GOLDY_ERR_INVALID_ARG, "bad element-wise descriptor");
+  goldy_status st = check_desc(*gemm, 0);
+  if (st != GOLDY_OK) return st;
+  const LutEntry& e = lookup(*lut, bucket_key(*gemm));
+  bool concurrent = false;
+  int variant = e.variant[0], add_rc_div = 1;
+  switch (policy) {
+    case GOLDY_PLAN_SEQUENTIAL: break;
+    case GOLDY_PLAN_DEFAULT: concurrent = true; break;
+    case GOLDY_PLAN_GO:
+      concurrent = true;
+      variant = e.variant[1];
+      add_rc_div = 2;
+      break;
+    default:   // the table's profiled configuration
+      if (e.flags & 1u) {
+        concurrent = true;
+        variant = (e.flags & 2u) ? e.variant[1] : e.variant[0];
+        add_rc_div = 1 << ((e.flags >> 2) & 3u);
+      }
+  }
+  const int group = 0, slot = 0;
+  goldy_schedule* s = nullptr;
+  st = goldy_schedule_build(gemm, 1, &group, &variant, &slot, 0, &s);
+  if (st != GOLDY_OK) return st;
+  goldy_corun* c = new (std::nothrow) goldy_corun();
+  if (!c) {
+    goldy_schedule_free(s);
+    return fail(GOLDY_ERR_NOMEM, "out of host memory");
+  }
+  c->gemm = s;
+  c->ew = *ew;
+  c->policy = policy;
+  c->concurrent = concurrent ? 1 : 0;
+  c->add_rc_div = add_rc_div;
+  *out = c;
+  return ok();
+}
+
+extern "C" goldy_status goldy_corun_query(const goldy_corun* c, int* concurrent, int* gemm_variant, int* add_rc_div,
+                                          size_t* workspace_bytes) {
+  if (!c) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  if (concurrent) *concurrent = c->concurrent;
+  if (gemm_variant) *gemm_variant = c->gemm->gemms[0].variant;
+  if (add_rc_div) *add_rc_div = c->add_rc_div;
+  if (workspace_bytes) *workspace_bytes = c->gemm->workspace_bytes;
+  return ok();
+}
+
+extern "C" void goldy_corun_free(goldy_corun* c) {
+  if (!c) return;
+  goldy_schedule_free(c->gemm);
+  goldy::runtime_release(c->rt);
+  delete c;
 }

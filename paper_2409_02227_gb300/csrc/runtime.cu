@@ -55,6 +55,7 @@ struct Op {
   cudaStream_t stream = nullptr;
   const void* fn = nullptr;
   unsigned grid = 0;
+  unsigned block = 0;
   size_t smem = 0;
   int cluster = 0;
   std::vector<uint64_t> params;      // 8-byte-aligned copy of the parameter block
@@ -158,9 +159,9 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
 // Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
 // cluster > 1.
 cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params,
-                              int cluster) {
+                              int cluster, unsigned block = kThreads) {
   void* args[] = {params};
-  if (cluster <= 1) return cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream);
+  if (cluster <= 1) return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
@@ -186,6 +187,23 @@ cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream
   op.grid = grid;
   op.smem = smem;
   op.cluster = cluster;
+  op.params.resize((params_size + 7) / 8);
+  std::memcpy(op.params.data(), params, params_size);
+  t_rec->push_back(std::move(op));
+  return cudaSuccess;
+}
+
+// A kernel with `block` threads per CTA and no cluster (recorded like launch_kernel).
+cudaError_t launch_kernel_threads(const void* fn, unsigned grid, unsigned block, size_t smem, cudaStream_t stream,
+                                  const void* params, size_t params_size) {
+  if (!t_rec) return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), 0, block);
+  Op op;
+  op.kind = Op::kKernel;
+  op.stream = stream;
+  op.fn = fn;
+  op.grid = grid;
+  op.block = block;
+  op.smem = smem;
   op.params.resize((params_size + 7) / 8);
   std::memcpy(op.params.data(), params, params_size);
   t_rec->push_back(std::move(op));
@@ -235,7 +253,7 @@ cudaError_t replay(const Op& op) {
   switch (op.kind) {
     case Op::kKernel:
       return launch_kernel_now(op.fn, op.grid, op.smem, op.stream, const_cast<uint64_t*>(op.params.data()),
-                               op.cluster);
+                               op.cluster, op.block ? op.block : kThreads);
     case Op::kMemset2D: return cudaMemset2DAsync(op.ptr, op.pitch, 0, op.width, op.height, op.stream);
     case Op::kEventRecord: return cudaEventRecord(op.ev, op.stream);
     case Op::kEventRecordExternal: return cudaEventRecordWithFlags(op.ev, op.stream, 0);
@@ -283,14 +301,17 @@ unsigned pair_grid(int64_t units, int64_t cap) {
   return unsigned(2 * pairs);
 }
 
-goldy_status encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-                       uint32_t box_inner, uint32_t box_outer,
+// Tensor map of a (batch x outer x inner) array: rows of `row_bytes`, batch
+// entries `batch_bytes` apart; boxes of box_outer rows x box_inner elements
+// of one entry, 128-byte swizzled.
+goldy_status encode_3d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t batch,
+                       uint64_t row_bytes, uint64_t batch_bytes, uint32_t box_inner, uint32_t box_outer,
                        CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
-  cuuint64_t dims[2] = {inner, outer};
-  cuuint64_t strides[1] = {row_bytes};
-  cuuint32_t box[2] = {box_inner, box_outer};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(m, dtype, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+  cuuint64_t dims[3] = {inner, outer, batch};
+  cuuint64_t strides[2] = {row_bytes, batch_bytes};
+  cuuint32_t box[3] = {box_inner, box_outer, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(m, dtype, 3, const_cast<void*>(ptr), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(GOLDY_ERR_CUDA, "cuTensorMapEncodeTiled failed with code " + std::to_string(int(r)));
@@ -305,14 +326,21 @@ goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const v
                        uint8_t* ws, int32_t unit_begin) {
   const goldy_gemm_desc& g = gp.desc;
   const KindInfo& k = kKinds[gp.kind];
-  goldy_status st =
-      encode_2d(&p.tmap_a[j], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.lda) * 2, kBlockK, uint32_t(a_box_rows(k)));
+  // batch strides in bytes; a single GEMM gets the packed stride (never read)
+  const bool batched = g.batch > 1;
+  const uint64_t sa = uint64_t(batched ? g.stride_a : g.M * g.lda) * 2;
+  const uint64_t sb = uint64_t(batched ? g.stride_b : g.K * g.ldb) * 2;
+  goldy_status st = encode_3d(&p.tmap_a[j], A, uint64_t(g.K), uint64_t(g.M), uint64_t(g.batch), uint64_t(g.lda) * 2,
+                              sa, kBlockK, uint32_t(a_box_rows(k)));
   if (st != GOLDY_OK) return st;
-  st = encode_2d(&p.tmap_b[j], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.ldb) * 2, 64, kBlockK);
+  st = encode_3d(&p.tmap_b[j], B, uint64_t(g.N), uint64_t(g.K), uint64_t(g.batch), uint64_t(g.ldb) * 2, sb, 64,
+                 kBlockK);
   if (st != GOLDY_OK) return st;
   GemmWork& w = p.g[j];
   w.c = C;
   w.ldc = g.ldc;
+  w.batch = int32_t(g.batch);
+  w.c_bstride = batched ? g.stride_c : g.M * g.ldc;
   w.m = int32_t(g.M);
   w.n = int32_t(g.N);
   w.k = int32_t(g.K);
@@ -325,8 +353,10 @@ goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const v
   // and rows; the epilogue writes 128-byte rows (32 fp32 / 64 bf16 columns)
   const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
   w.c_tma = 0;
-  if (epi_tma(k) && gp.split == 1 && aligned(C, 16) && (size_t(g.ldc) * es) % 16 == 0) {
-    st = encode_2d(&p.tmap_c[j], C, uint64_t(g.N), uint64_t(g.M), uint64_t(g.ldc) * es, uint32_t(128 / es), 128,
+  const uint64_t sc = uint64_t(w.c_bstride) * es;
+  if (epi_tma(k) && gp.split == 1 && aligned(C, 16) && (size_t(g.ldc) * es) % 16 == 0 && sc % 16 == 0) {
+    st = encode_3d(&p.tmap_c[j], C, uint64_t(g.N), uint64_t(g.M), uint64_t(g.batch), uint64_t(g.ldc) * es, sc,
+                   uint32_t(128 / es), 128,
                    g.c_dtype == GOLDY_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
     if (st != GOLDY_OK) return st;
     w.c_tma = 1;
@@ -345,8 +375,17 @@ goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream)
   const goldy_gemm_desc& g = gp.desc;
   if (g.M == 0 || g.N == 0) return GOLDY_OK;
   const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
-  cudaError_t e = enq_memset2d(C, size_t(g.ldc) * es, size_t(g.N) * es, size_t(g.M), stream);
-  return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
+  const int64_t cstride = g.batch > 1 ? g.stride_c : g.M * g.ldc;
+  if (cstride == g.M * g.ldc) {   // entries packed: one 2-D fill over all of them
+    cudaError_t e = enq_memset2d(C, size_t(g.ldc) * es, size_t(g.N) * es, size_t(g.M * g.batch), stream);
+    return e == cudaSuccess ? GOLDY_OK : cuda_fail(e, "cudaMemset2DAsync");
+  }
+  for (int64_t b = 0; b < g.batch; ++b) {
+    cudaError_t e = enq_memset2d(static_cast<char*>(C) + size_t(b * cstride) * es, size_t(g.ldc) * es,
+                                 size_t(g.N) * es, size_t(g.M), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemset2DAsync");
+  }
+  return GOLDY_OK;
 }
 
 // Phase-trace buffer of the current goldy_run_ex call (null: off).
@@ -747,6 +786,7 @@ extern "C" goldy_status goldy_run_ex(const goldy_schedule* s, const void* const*
 struct goldy_exec {
   std::vector<Op> ops;
   Runtime* rt = nullptr;
+  Runtime* rt2 = nullptr;    // a co-run's own fork/join events
   CUcontext ctx = nullptr;   // the partition's context to make current while replaying (null: none)
   cudaStream_t main = nullptr;
 };
@@ -841,7 +881,153 @@ extern "C" goldy_status goldy_exec_time(const goldy_exec* const* execs, int n, i
 extern "C" void goldy_exec_free(goldy_exec* x) {
   if (!x) return;
   runtime_release(x->rt);
+  runtime_release(x->rt2);
   delete x;
+}
+
+// ---------------------------------------------------------------------------
+// Element-wise add and a GEMM co-scheduled with it
+// ---------------------------------------------------------------------------
+static goldy_status launch_ewise(const DeviceState& d, const goldy_ewise_desc& ew, const void* X, const void* Y,
+                                 void* Z, int rc_div, cudaStream_t stream) {
+  if (ew.n == 0) return GOLDY_OK;
+  EwiseParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.x = X;
+  p.y = Y;
+  p.z = Z;
+  p.n = ew.n;
+  p.vec_ok = (aligned(X, 16) && aligned(Y, 16) && aligned(Z, 16)) ? 1 : 0;
+  const int64_t per_vec = ew.dtype == GOLDY_BF16 ? 8 : 4;
+  const int64_t work = p.vec_ok ? (ew.n + per_vec - 1) / per_vec : ew.n;
+  const int64_t cap = std::max<int64_t>(1, int64_t(kEwiseCtasPerSm) * sms(d) / rc_div);
+  const unsigned grid = unsigned(std::max<int64_t>(1, std::min<int64_t>(cap, (work + kEwiseThreads - 1) / kEwiseThreads)));
+  cudaError_t e = launch_kernel_threads(ewise_kernel_fn(ew.dtype == GOLDY_BF16 ? 1 : 0), grid, kEwiseThreads, 0,
+                                        stream, &p, sizeof(p));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaLaunchKernel (element-wise add)");
+  return GOLDY_OK;
+}
+
+static goldy_status check_ewise(const goldy_ewise_desc& ew, const void* X, const void* Y, void* Z, int rc_div) {
+  if (ew.n < 0 || ew.reserved != 0 || (ew.dtype != GOLDY_BF16 && ew.dtype != GOLDY_F32))
+    return fail(GOLDY_ERR_INVALID_ARG, "bad element-wise descriptor");
+  if (rc_div != 1 && rc_div != 2 && rc_div != 4) return fail(GOLDY_ERR_INVALID_ARG, "rc_div must be 1, 2 or 4");
+  const size_t es = ew.dtype == GOLDY_BF16 ? 2 : 4;
+  if (ew.n > 0 && (!X || !Y || !Z || !aligned(X, es) || !aligned(Y, es) || !aligned(Z, es)))
+    return fail(GOLDY_ERR_INVALID_ARG, "element-wise operands null or misaligned");
+  return GOLDY_OK;
+}
+
+extern "C" goldy_status goldy_ewise_add(const void* X, const void* Y, void* Z, int64_t n, int dtype, int rc_div,
+                                        void* stream) {
+  goldy_ewise_desc ew{n, dtype, 0};
+  goldy_status st = check_ewise(ew, X, Y, Z, rc_div);
+  if (st != GOLDY_OK) return st;
+  DeviceState* d = nullptr;
+  st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+  PartitionScope part;
+  st = part.enter(stream);
+  if (st != GOLDY_OK) return st;
+  st = launch_ewise(*d, ew, X, Y, Z, rc_div, static_cast<cudaStream_t>(stream));
+  return st == GOLDY_OK ? ok() : st;
+}
+
+// gemm_rt: events of the GEMM's run (null: the GEMM schedule's own);
+// corun_rt: the fork/join events of the two streams (null: the co-run's own).
+static goldy_status corun_impl(const goldy_corun* c, const void* A, const void* B, void* C, void* ws,
+                               size_t ws_bytes, const void* X, const void* Y, void* Z, void* const* streams,
+                               int n_streams, Runtime* gemm_rt, Runtime* corun_rt) {
+  if (!c || !streams) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  if (n_streams < (c->concurrent ? 2 : 1)) return fail(GOLDY_ERR_INVALID_ARG, "fewer streams than the co-run needs");
+  goldy_status st = check_ewise(c->ew, X, Y, Z, c->add_rc_div);
+  if (st != GOLDY_OK) return st;
+  DeviceState* d = nullptr;
+  st = device_state(&d);
+  if (st != GOLDY_OK) return st;
+  PartitionScope part;
+  st = part.enter(streams[0]);
+  if (st != GOLDY_OK) return st;
+  cudaStream_t s0 = static_cast<cudaStream_t>(streams[0]);
+  const void* const a[1] = {A};
+  const void* const b[1] = {B};
+  void* const cc[1] = {C};
+  if (!c->concurrent) {
+    st = run_impl(c->gemm, a, b, cc, ws, ws_bytes, streams, 1, nullptr, gemm_rt);
+    if (st != GOLDY_OK) return st;
+    st = launch_ewise(*d, c->ew, X, Y, Z, c->add_rc_div, s0);
+    return st == GOLDY_OK ? ok() : st;
+  }
+  Runtime* rt = corun_rt;
+  if (!rt) {
+    goldy_corun* mc = const_cast<goldy_corun*>(c);
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (mc->rt && (mc->rt->device != dev || mc->rt->green != part.green())) {
+      runtime_release(mc->rt);
+      mc->rt = nullptr;
+    }
+    if (!mc->rt) {
+      mc->rt = new_runtime(dev, part.green(), &st);
+      if (!mc->rt) return st;
+    }
+    rt = mc->rt;
+  }
+  cudaStream_t s1 = static_cast<cudaStream_t>(streams[1]);
+  cudaError_t e = enq_event_record(rt->fork, s0);
+  if (e == cudaSuccess) e = enq_wait(s1, rt->fork);
+  if (e != cudaSuccess) return cuda_fail(e, "co-run fork");
+  st = run_impl(c->gemm, a, b, cc, ws, ws_bytes, streams, 1, nullptr, gemm_rt);
+  if (st != GOLDY_OK) return st;
+  st = launch_ewise(*d, c->ew, X, Y, Z, c->add_rc_div, s1);
+  if (st != GOLDY_OK) return st;
+  e = enq_event_record(rt->join[0], s1);
+  if (e == cudaSuccess) e = enq_wait(s0, rt->join[0]);
+  if (e != cudaSuccess) return cuda_fail(e, "co-run join");
+  return ok();
+}
+
+extern "C" goldy_status goldy_corun_run(const goldy_corun* c, const void* A, const void* B, void* C, void* workspace,
+                                        size_t workspace_bytes, const void* X, const void* Y, void* Z,
+                                        void* const* streams, int n_streams) {
+  return corun_impl(c, A, B, C, workspace, workspace_bytes, X, Y, Z, streams, n_streams, nullptr, nullptr);
+}
+
+extern "C" goldy_status goldy_corun_exec_create(const goldy_corun* c, const void* A, const void* B, void* C,
+                                                void* workspace, size_t workspace_bytes, const void* X,
+                                                const void* Y, void* Z, void* const* streams, int n_streams,
+                                                goldy_exec** out) {
+  if (!out || !c || !streams || n_streams < 1) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  int dev = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce != cudaSuccess) return cuda_fail(ce, "cudaGetDevice");
+  PartitionScope part;
+  goldy_status st = part.enter(streams[0]);
+  if (st != GOLDY_OK) return st;
+  goldy_exec* x = new (std::nothrow) goldy_exec();
+  if (!x) return fail(GOLDY_ERR_NOMEM, "out of host memory");
+  if (part.green() && green_api().to_ctx(&x->ctx, static_cast<CUgreenCtx>(part.green())) != CUDA_SUCCESS) {
+    delete x;
+    return fail(GOLDY_ERR_CUDA, "cuCtxFromGreenCtx failed");
+  }
+  x->main = static_cast<cudaStream_t>(streams[0]);
+  x->rt = new_runtime(dev, part.green(), &st);
+  if (x->rt) x->rt2 = new_runtime(dev, part.green(), &st);
+  if (!x->rt || !x->rt2) {
+    goldy_exec_free(x);
+    return st;
+  }
+  t_rec = &x->ops;
+  st = corun_impl(c, A, B, C, workspace, workspace_bytes, X, Y, Z, streams, n_streams, x->rt, x->rt2);
+  t_rec = nullptr;
+  if (st != GOLDY_OK) {
+    std::string why = goldy_last_error();
+    goldy_exec_free(x);
+    return fail(st, why);
+  }
+  *out = x;
+  return ok();
 }
 
 struct goldy_graph {

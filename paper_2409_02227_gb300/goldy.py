@@ -51,12 +51,18 @@ class GoldyError(RuntimeError):
         self.status = status
 
 
+class goldy_ewise_desc(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 class goldy_gemm_desc(ctypes.Structure):
     _fields_ = [("M", ctypes.c_int64), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
                 ("lda", ctypes.c_int64), ("ldb", ctypes.c_int64), ("ldc", ctypes.c_int64),
                 ("trans_a", ctypes.c_int32), ("trans_b", ctypes.c_int32),
                 ("a_dtype", ctypes.c_int32), ("b_dtype", ctypes.c_int32),
-                ("c_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("c_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("batch", ctypes.c_int64), ("stride_a", ctypes.c_int64), ("stride_b", ctypes.c_int64),
+                ("stride_c", ctypes.c_int64)]
 
 
 class goldy_run_opts(ctypes.Structure):
@@ -115,6 +121,12 @@ def _load():
         "goldy_exec_launch": ([P], I),
         "goldy_exec_time": ([PP, I, I, I, ctypes.POINTER(ctypes.c_float)], I),
         "goldy_partition_create": ([I, I, PP], I),
+        "goldy_corun_plan": ([DP, ctypes.POINTER(goldy_ewise_desc), P, I, PP], I),
+        "goldy_corun_query": ([P, IP, IP, IP, ctypes.POINTER(SZ)], I),
+        "goldy_corun_run": ([P, P, P, P, P, SZ, P, P, P, PP, I], I),
+        "goldy_corun_exec_create": ([P, P, P, P, P, SZ, P, P, P, PP, I, PP], I),
+        "goldy_corun_free": ([P], None),
+        "goldy_ewise_add": ([P, P, P, ctypes.c_int64, I, I, P], I),
         "goldy_partition_query": ([P, IP, PP, I], I),
         "goldy_partition_free": ([P], None),
         "goldy_exec_free": ([P], None),
@@ -153,10 +165,17 @@ def _descs(descs: Sequence[goldy_gemm_desc]):
 
 
 def desc(M: int, N: int, K: int, c_dtype: int = GOLDY_F32, lda: Optional[int] = None,
-         ldb: Optional[int] = None, ldc: Optional[int] = None) -> goldy_gemm_desc:
-    """Descriptor of C (M x N) = A (M x K, row-major) * B (K x N, row-major)."""
-    return goldy_gemm_desc(M, N, K, K if lda is None else lda, N if ldb is None else ldb,
-                           N if ldc is None else ldc, 0, 0, GOLDY_BF16, GOLDY_BF16, int(c_dtype), 0)
+         ldb: Optional[int] = None, ldc: Optional[int] = None, batch: int = 1, stride_a: Optional[int] = None,
+         stride_b: Optional[int] = None, stride_c: Optional[int] = None) -> goldy_gemm_desc:
+    """Descriptor of C (M x N) = A (M x K, row-major) * B (K x N, row-major),
+    or of `batch` such products with entries packed back to back (default
+    strides M*lda, K*ldb, M*ldc)."""
+    lda = K if lda is None else lda
+    ldb = N if ldb is None else ldb
+    ldc = N if ldc is None else ldc
+    return goldy_gemm_desc(M, N, K, lda, ldb, ldc, 0, 0, GOLDY_BF16, GOLDY_BF16, int(c_dtype), 0, int(batch),
+                           M * lda if stride_a is None else stride_a, K * ldb if stride_b is None else stride_b,
+                           M * ldc if stride_c is None else stride_c)
 
 
 class _Handle:
@@ -191,6 +210,10 @@ class Schedule(_Handle):
 
 class Graph(_Handle):
     _free = staticmethod(lambda p: _lib.goldy_graph_free(p))
+
+
+class Corun(_Handle):
+    _free = staticmethod(lambda p: _lib.goldy_corun_free(p))
 
 
 class Partition(_Handle):
@@ -393,6 +416,43 @@ def goldy_exec_time(execs: Sequence[Exec], warmup: int, reps: int) -> float:
     ms = ctypes.c_float()
     _check(_lib.goldy_exec_time(arr, len(execs), int(warmup), int(reps), ctypes.byref(ms)), "goldy_exec_time")
     return ms.value
+
+
+def goldy_corun_plan(gemm: goldy_gemm_desc, n: int, dtype: int, lut: Lut, policy: int = GOLDY_PLAN_AUTO) -> Corun:
+    """A GEMM co-scheduled with the element-wise add Z = X + Y of n elements."""
+    ew = goldy_ewise_desc(int(n), int(dtype), 0)
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_corun_plan(ctypes.byref(gemm), ctypes.byref(ew), lut.ptr if lut else None, int(policy),
+                                 ctypes.byref(out)), "goldy_corun_plan")
+    return Corun(out)
+
+
+def goldy_corun_query(c: Corun) -> Tuple[int, int, int, int]:
+    """(concurrent, gemm variant, add grid-cap divisor, workspace bytes)."""
+    cc, v, rc, ws = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_size_t()
+    _check(_lib.goldy_corun_query(c.ptr, ctypes.byref(cc), ctypes.byref(v), ctypes.byref(rc), ctypes.byref(ws)),
+           "goldy_corun_query")
+    return cc.value, v.value, rc.value, ws.value
+
+
+def goldy_corun_run(c: Corun, A: int, B: int, C: int, workspace: int, workspace_bytes: int, X: int, Y: int, Z: int,
+                    streams: Sequence[int]) -> None:
+    _check(_lib.goldy_corun_run(c.ptr, A or None, B or None, C or None, workspace or None, int(workspace_bytes),
+                                X or None, Y or None, Z or None, _ptrs(streams), len(streams)), "goldy_corun_run")
+
+
+def goldy_corun_exec_create(c: Corun, A: int, B: int, C: int, workspace: int, workspace_bytes: int, X: int, Y: int,
+                            Z: int, streams: Sequence[int]) -> "Exec":
+    out = ctypes.c_void_p()
+    _check(_lib.goldy_corun_exec_create(c.ptr, A or None, B or None, C or None, workspace or None,
+                                        int(workspace_bytes), X or None, Y or None, Z or None, _ptrs(streams),
+                                        len(streams), ctypes.byref(out)), "goldy_corun_exec_create")
+    return Exec(out)
+
+
+def goldy_ewise_add(X: int, Y: int, Z: int, n: int, dtype: int, rc_div: int, stream: int) -> None:
+    _check(_lib.goldy_ewise_add(X or None, Y or None, Z or None, int(n), int(dtype), int(rc_div), stream or None),
+           "goldy_ewise_add")
 
 
 def goldy_partition_create(min_sms: int, n_streams: int = 16) -> Partition:

@@ -25,7 +25,9 @@ Each bucket (floor log2 of M, N, K; output dtype) is profiled at its lower
 edge (M, N, K = powers of two), where DNN layer sizes usually sit.  Timing:
 prepared runs (recorded plain launches, the way the benchmark replays a step)
 back to back on one stream, as the paper ran GEMMs back to back on each
-stream (Sec. 5.3); the median of several repetitions of a timed batch.
+stream (Sec. 5.3), rotating over disjoint copies of the operands so that they
+come from HBM as in the benchmark (inputs rotated past twice the L2); the
+median of several repetitions of a timed batch.
 Results are appended to a JSONL log bucket by bucket, so an interrupted run
 resumes where it stopped; the LUT file is written at the end.
 
@@ -61,13 +63,15 @@ NONSWAP_KINDS = (0, 1, 2, 3, 4, 5)
 PAIR_KINDS = (10,)
 
 
-def write_lut(entries: Sequence[Tuple[Tuple[int, int, int, int], int, Sequence[int]]],
-              n_variants: int, sm_count: int) -> bytes:
-    """LUT bytes in the format goldy_lut_load reads (include/goldy.h)."""
+def write_lut(entries, n_variants: int, sm_count: int) -> bytes:
+    """LUT bytes in the format goldy_lut_load reads (include/goldy.h) from
+    (key, preferred CD, variants[, flags]) tuples."""
     out = bytearray(b"GOLDYLUT")
     out += struct.pack("<IIIIII", 1, len(entries), n_variants, sm_count, 0, 0)
-    for key, pref, variants in sorted(entries, key=lambda e: e[0]):
-        out += bytes([key[0], key[1], key[2], key[3], pref, 0])
+    for e in sorted(entries, key=lambda e: e[0]):
+        key, pref, variants = e[0], e[1], e[2]
+        flags = e[3] if len(e) > 3 else 0
+        out += bytes([key[0], key[1], key[2], key[3], pref, flags])
         out += struct.pack("<5H", *variants)
     return bytes(out)
 
@@ -110,19 +114,31 @@ def candidates(M: int, N: int, K: int, sm_count: int) -> List[Tuple[int, int]]:
 
 
 class Bench:
-    """Buffers for up to 16 copies of one GEMM, timed through graph replays."""
+    """Device copies of one GEMM, timed as prepared runs replayed back to back
+    on the bench's streams (or a partition's).  A co-run of c copies is
+    prepared once per disjoint group of c copies and the replays rotate over
+    the groups, so that — as in the benchmark — the inputs touched between
+    two uses of the same copy exceed twice the L2 and every GEMM reads its
+    operands from HBM."""
 
     def __init__(self, M: int, N: int, K: int, out: int, copies: int = 16, seed: int = 0, partition=None,
-                 graph_replay: bool = False):
+                 rotate: bool = True, max_bytes: int = 6 << 30):
         self.M, self.N, self.K, self.out = M, N, K, out
         self.partition = partition
-        self.graph_replay = graph_replay
+        cdt = torch.float32 if out == G.GOLDY_F32 else torch.bfloat16
+        per = 2 * M * K + 2 * K * N
+        cbytes = M * N * (4 if out == G.GOLDY_F32 else 2)
+        l2 = int(getattr(torch.cuda.get_device_properties(torch.cuda.current_device()), "L2_cache_size", 126 << 20))
+        total = copies
+        if rotate:
+            total = max(copies, -(-2 * l2 // max(per, 1)) + copies)
+            total = min(total, max(copies, max_bytes // max(per + cbytes, 1)))
+        self.total = total
         gen = torch.Generator(device="cuda")
         gen.manual_seed(seed)
-        cdt = torch.float32 if out == G.GOLDY_F32 else torch.bfloat16
-        self.A = [(torch.rand((M, K), generator=gen, device="cuda") - 0.5).to(torch.bfloat16) for _ in range(copies)]
-        self.B = [(torch.rand((K, N), generator=gen, device="cuda") - 0.5).to(torch.bfloat16) for _ in range(copies)]
-        self.C = [torch.empty((M, N), dtype=cdt, device="cuda") for _ in range(copies)]
+        self.A = [(torch.rand((M, K), generator=gen, device="cuda") - 0.5).to(torch.bfloat16) for _ in range(total)]
+        self.B = [(torch.rand((K, N), generator=gen, device="cuda") - 0.5).to(torch.bfloat16) for _ in range(total)]
+        self.C = [torch.empty((M, N), dtype=cdt, device="cuda") for _ in range(total)]
         self.streams = [torch.cuda.Stream() for _ in range(16)]
         self.part_streams = (G.goldy_partition_query(partition, 16)[1] if partition is not None
                              else [st.cuda_stream for st in self.streams])
@@ -135,6 +151,8 @@ class Bench:
 
     def time_us(self, variant: int, copies: int, concurrent: bool, target_us: float = 2000.0,
                 fused: bool = True, samples: int = 5) -> float:
+        """Median time of one co-run of `copies` GEMMs with `variant` (samples
+        = 0: quick mode, a single replay when it alone reaches target_us)."""
         d = G.desc(self.M, self.N, self.K, self.out)
         slots = list(range(copies)) if concurrent else [0] * copies
         sched = G.goldy_schedule_build([d] * copies, [0] * copies, [variant] * copies, slots,
@@ -142,37 +160,25 @@ class Bench:
         _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
         ws = self._workspace(ws_bytes)
         torch.cuda.synchronize()
-        if not self.graph_replay:
-            return self._time_exec(sched, copies, ws, ws_bytes, ms, target_us, samples)
-        g = G.goldy_graph_create(sched, [a.data_ptr() for a in self.A[:copies]],
-                                 [b.data_ptr() for b in self.B[:copies]],
-                                 [c.data_ptr() for c in self.C[:copies]], ws.data_ptr(), ws_bytes,
-                                 [s.cuda_stream for s in self.streams[:max(1, ms)]])
-        main = self.streams[0]
-        for _ in range(3 if samples else 1):
-            G.goldy_graph_launch(g, main.cuda_stream)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(main)
-        G.goldy_graph_launch(g, main.cuda_stream)
-        e1.record(main)
-        torch.cuda.synchronize()
-        est = max(e0.elapsed_time(e1) * 1e3, 1.0)
-        if samples == 0:                 # quick mode: one replay is long enough to time on its own
+        groups = max(1, self.total // copies)
+        execs = []
+        for r in range(groups):
+            lo, hi = r * copies, (r + 1) * copies
+            execs.append(G.goldy_exec_create(sched, [a.data_ptr() for a in self.A[lo:hi]],
+                                             [b.data_ptr() for b in self.B[lo:hi]],
+                                             [c.data_ptr() for c in self.C[lo:hi]], ws.data_ptr(), ws_bytes,
+                                             self.part_streams[:max(1, ms)]))
+        est = max(G.goldy_exec_time(execs, min(groups, 3 if samples else 1), 1) * 1e3, 1.0)
+        if samples == 0:
             if est >= target_us:
+                del execs
                 return est
             samples = 3
-        reps = int(min(200, max(3, target_us / est)))
-        times = []
-        for _ in range(samples):
-            e0.record(main)
-            for _ in range(reps):
-                G.goldy_graph_launch(g, main.cuda_stream)
-            e1.record(main)
-            torch.cuda.synchronize()
-            times.append(e0.elapsed_time(e1) * 1e3 / reps)
+        reps = int(min(2000, max(3, target_us / est)))
+        times = sorted(G.goldy_exec_time(execs, 0, reps) * 1e3 for _ in range(samples))
+        del execs
         if G.goldy_device_error(clear=True) != 0:
             raise RuntimeError("kernel reported a bounded-wait timeout while profiling")
-        times.sort()
         return times[len(times) // 2]
 
 
@@ -215,27 +221,92 @@ def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) 
     return rec
 
 
-def _time_exec(self, sched, copies, ws, ws_bytes, ms, target_us, samples):
-    """time_us as prepared runs (recorded plain launches) replayed back to back
-    on the bench's streams — or the partition's — and timed by events on the
-    first of them (goldy_exec_time)."""
-    x = G.goldy_exec_create(sched, [a.data_ptr() for a in self.A[:copies]], [b.data_ptr() for b in self.B[:copies]],
-                            [c.data_ptr() for c in self.C[:copies]], ws.data_ptr(), ws_bytes,
-                            self.part_streams[:max(1, ms)])
-    est = max(G.goldy_exec_time([x], 3 if samples else 1, 1) * 1e3, 1.0)
-    if samples == 0:
-        if est >= target_us:
-            return est
-        samples = 3
-    reps = int(min(200, max(3, target_us / est)))
-    times = sorted(G.goldy_exec_time([x], 0, reps) * 1e3 for _ in range(samples))
-    del x
+
+
+
+CORUN_CONFIGS = [(f"v{vi}_rc{1 << ri}", 1 | (vi << 1) | (ri << 2)) for vi in (0, 1) for ri in (0, 1, 2)]
+
+
+def corun_times(bench: "Bench", variants: Sequence[int], target_us: float = 2000.0) -> Dict[str, float]:
+    """Step 3 (Sec. 8.1): the bucket's GEMM with an element-wise add of its
+    output size, one after the other ("sequential": the CD-1 kernel, then the
+    add over the whole GPU) and at once in every configuration the table can
+    record: the CD-1 or the CD-2 GO-Kernel ("v0", "v1") with the add's grid
+    capped at GPU, GPU/2 or GPU/4 ("rc1", "rc2", "rc4").  Rotates over the
+    bench's copies like time_us."""
+    M, N, K, out = bench.M, bench.N, bench.K, bench.out
+    n = M * N
+    cdt = torch.float32 if out == G.GOLDY_F32 else torch.bfloat16
+    R = max(1, bench.total // 2)              # the add's operands double the bytes per copy
+    if getattr(bench, "X", None) is None:
+        bench.X = [torch.randn(n, device="cuda").to(cdt) for _ in range(R)]
+        bench.Y = [torch.randn(n, device="cuda").to(cdt) for _ in range(R)]
+        bench.Z = [torch.empty(n, device="cuda", dtype=cdt) for _ in range(R)]
+    streams = bench.part_streams[:2]
+    t = {}
+    for name, flags in [("sequential", 0)] + CORUN_CONFIGS:
+        lut = G.goldy_lut_from_memory(write_lut([((0, 0, 0, out), 2, list(variants), flags)],
+                                                G.goldy_variant_count(), 0))
+        c = G.goldy_corun_plan(G.desc(M, N, K, out), n, out, lut, G.GOLDY_PLAN_AUTO)
+        _, _, _, ws_bytes = G.goldy_corun_query(c)
+        ws = bench._workspace(ws_bytes)
+        torch.cuda.synchronize()
+        execs = [G.goldy_corun_exec_create(c, bench.A[r].data_ptr(), bench.B[r].data_ptr(), bench.C[r].data_ptr(),
+                                           ws.data_ptr(), ws_bytes, bench.X[r].data_ptr(), bench.Y[r].data_ptr(),
+                                           bench.Z[r].data_ptr(), streams) for r in range(R)]
+        est = max(G.goldy_exec_time(execs, min(R, 3), 1) * 1e3, 1.0)
+        reps = int(min(2000, max(3, target_us / est)))
+        t[name] = sorted(G.goldy_exec_time(execs, 0, reps) * 1e3 for _ in range(5))[2]
+        del execs
     if G.goldy_device_error(clear=True) != 0:
         raise RuntimeError("kernel reported a bounded-wait timeout while profiling")
-    return times[len(times) // 2]
+    return t
 
 
-Bench._time_exec = _time_exec
+def corun_flags(t: Dict[str, float], gain: float = 0.05) -> int:
+    """The table's co-run flags from step 3's times: the fastest configuration
+    at once, taken only when it beats one after the other by `gain` (the
+    preferred-CD rule's threshold, Sec. 5.4); 0 (sequential) otherwise."""
+    name, flags = min(CORUN_CONFIGS, key=lambda c: (t[c[0]], c[1]))
+    return flags if t[name] * (1.0 + gain) <= t["sequential"] else 0
+
+
+def add_corun_flags(out_dir: str, fused: bool, partition=None) -> None:
+    """Step 3 over a profiled table: time every bucket's GEMM + element-wise
+    add in each configuration and record the chosen one in the entry's flags."""
+    prof = os.path.join(out_dir, "profile.jsonl")
+    recs = {}
+    for line in open(prof):
+        r = json.loads(line)
+        recs[tuple(r["key"])] = r
+    log_path = os.path.join(out_dir, "corun.jsonl")
+    done = {}
+    if os.path.exists(log_path):
+        for line in open(log_path):
+            r = json.loads(line)
+            done[tuple(r["key"])] = r
+    with open(log_path, "a") as log:
+        for i, (key, r) in enumerate(sorted(recs.items())):
+            if key in done:
+                continue
+            M, N, K, out = bucket_shape(key)
+            bench = Bench(M, N, K, out, copies=2, partition=partition)
+            t = corun_times(bench, r["variants"])
+            rec = {"key": list(key), "shape": [M, N, K, out], "t_us": t, "flags": corun_flags(t)}
+            log.write(json.dumps(rec) + "\n")
+            log.flush()
+            done[key] = rec
+            del bench
+            torch.cuda.empty_cache()
+            if i % 20 == 0:
+                print(f"[corun {i + 1}/{len(recs)}] {key} {t}", flush=True)
+    sm_count = struct.unpack_from("<I", open(os.path.join(out_dir, "goldy_lut.bin"), "rb").read(), 20)[0]
+    entries = [(k, r["pref_cd"], r["variants"], done[k]["flags"]) for k, r in recs.items()]
+    lut = write_lut(entries, G.goldy_variant_count(), sm_count)
+    G.goldy_lut_from_memory(lut)
+    with open(os.path.join(out_dir, "goldy_lut.bin"), "wb") as f:
+        f.write(lut)
+    print(f"co-run at once on {sum(1 for e in entries if e[3] & 1)} of {len(entries)} buckets", flush=True)
 
 
 def profile_dataset_gemm(shape, lut, log, fused: bool = True) -> dict:
@@ -311,6 +382,8 @@ def main(argv=None) -> int:
                     help="tune inside an SM partition (green context) of at least SMS SMs (0: the whole GPU "
                          "as a partition); grid caps and the table's SM count follow the partition")
     ap.add_argument("--scaling-keys", action="store_true", help="buckets of the GPU-scaling study's sets")
+    ap.add_argument("--corun-flags", action="store_true",
+                    help="step 3 over the table already profiled in --out: set each bucket's co-run flag")
     ap.add_argument("--configs", action="store_true", help="buckets of the fixed workload sets")
     ap.add_argument("--sweep", action="store_true", help="buckets of the 64 randomized sets")
     ap.add_argument("--keys", nargs="*", default=[], help="extra buckets lm,ln,lk,out")
@@ -322,6 +395,10 @@ def main(argv=None) -> int:
         return run_dataset(args.dataset, args.dataset_size, args.lut, args.launch == "fused", args.time_budget)
     if not args.out:
         ap.error("--out is required to build a table")
+    if args.corun_flags:
+        part = G.goldy_partition_create(args.partition, 16) if args.partition is not None else None
+        add_corun_flags(args.out, args.launch == "fused", part)
+        return 0
     os.makedirs(args.out, exist_ok=True)
     keys = []
     if args.configs:

@@ -21,6 +21,8 @@ families it describes:
 * ``sweep``       — 64 sets of 2-16 GEMMs, M log-uniform in [16, 4096],
                     N and K log-uniform in [256, 8192] rounded to multiples of
                     64, U[-1, 1], fp32 out; set j uses seed 1000 + j.
+* batched study   — sets of 2 or 4 strided-batched attention GEMMs over
+                    variable sequence lengths (``make_batched_set``).
 
 Drawing order (fixed, so a set is reproducible from its seed): for GEMM i in
 order, A_i (M x K) then B_i (K x N), each as fp32 values rounded to bf16
@@ -49,16 +51,17 @@ class GemmSpec:
     out_dtype: int              # DTYPE_BF16 or DTYPE_F32
     dist: str                   # "uniform" or "normal"
     scale: float                # half-width for uniform, std-dev for normal
+    batch: int = 1              # strided batch entries (A: batch x M x K, B: batch x K x N)
 
     @property
     def flops(self) -> int:
-        return 2 * self.M * self.N * self.K
+        return 2 * self.M * self.N * self.K * self.batch
 
     @property
     def bytes(self) -> int:
         """Algorithmic bytes: A and B read once, C written once."""
         out = 2 if self.out_dtype == DTYPE_BF16 else 4
-        return 2 * self.M * self.K + 2 * self.K * self.N + out * self.M * self.N
+        return self.batch * (2 * self.M * self.K + 2 * self.K * self.N + out * self.M * self.N)
 
 
 @dataclass
@@ -108,8 +111,16 @@ def materialize(name: str, seed: int, specs: List[GemmSpec],
         gen.manual_seed(seed)
     s = GemmSet(name, seed, list(specs))
     for sp in specs:
-        s.a.append(_draw(gen, sp.M, sp.K, sp.dist, sp.scale))
-        s.b.append(_draw(gen, sp.K, sp.N, sp.dist, sp.scale))
+        if sp.batch == 1:
+            s.a.append(_draw(gen, sp.M, sp.K, sp.dist, sp.scale))
+            s.b.append(_draw(gen, sp.K, sp.N, sp.dist, sp.scale))
+        else:   # entry by entry: A_i then B_i
+            a, b = [], []
+            for _ in range(sp.batch):
+                a.append(_draw(gen, sp.M, sp.K, sp.dist, sp.scale))
+                b.append(_draw(gen, sp.K, sp.N, sp.dist, sp.scale))
+            s.a.append(torch.stack(a))
+            s.b.append(torch.stack(b))
     return s
 
 
@@ -203,6 +214,33 @@ def make_scaling_set(i: int, copies: int = 4) -> GemmSet:
     M, N, K, out = scaling_study_shapes()[i]
     specs = [GemmSpec(M, N, K, out, "uniform", 1.0) for _ in range(copies)]
     return materialize(f"scaling_{i:02d}", 3000 + i, specs)
+
+
+def batched_study_specs(i: int, members: int) -> Tuple[int, List[GemmSpec]]:
+    """Set i of the batched study: `members` (2 or 4) heterogeneous strided
+    batched GEMMs of attention over variable-length inputs (Sec. 6.6's
+    B-GEMMs): per member a sequence length L from {128, ..., 2048} and 16 or
+    32 heads of dimension 128, as scores = Q K^T (M = L, N = L, K = 128) or
+    output = P V (M = L, N = 128, K = L), batch = heads; bf16 out,
+    N(0, 1/sqrt(K)) inputs, seed 6000 + 100 * members + i."""
+    seed = 6000 + 100 * members + i
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed)
+    specs = []
+    for _ in range(members):
+        L = 128 * (1 << int(torch.randint(0, 5, (1,), generator=gen)[0]))
+        heads = 16 * (1 + int(torch.randint(0, 2, (1,), generator=gen)[0]))
+        if int(torch.randint(0, 2, (1,), generator=gen)[0]) == 0:
+            M, N, K = L, L, 128
+        else:
+            M, N, K = L, 128, L
+        specs.append(GemmSpec(M, N, K, DTYPE_BF16, "normal", 1.0 / math.sqrt(K), heads))
+    return seed, specs
+
+
+def make_batched_set(i: int, members: int) -> GemmSet:
+    seed, specs = batched_study_specs(i, members)
+    return materialize(f"bgemm{members}_{i:02d}", seed, specs)
 
 
 def make_sweep_set(j: int) -> GemmSet:

@@ -31,6 +31,11 @@ def test_lut_writer_matches_oracle_format():
     ref = pr.write_lut([pr.Entry(k, p, tuple(v)) for k, p, v in entries], 120, 152)
     assert mine == ref
     G.goldy_lut_from_memory(mine)
+    # with the co-run flag of step 3
+    flagged = [(k, p, v, rng.randint(0, 3) | (rng.randint(0, 2) << 2)) for k, p, v in entries]
+    mine = P.write_lut(flagged, 120, 152)
+    assert mine == pr.write_lut([pr.Entry(k, p, tuple(v), f) for k, p, v, f in flagged], 120, 152)
+    G.goldy_lut_from_memory(mine)
 
 
 def test_bucket_shapes_and_candidates():
@@ -76,3 +81,22 @@ def test_multi_rank_max_over_gloo():
         p.join(timeout=60)
         assert p.exitcode == 0
     assert res == {0: 11.0, 1: 11.0}
+
+
+def test_corun_flags_rule():
+    base = {"sequential": 10.0, "v0_rc1": 9.9, "v0_rc2": 9.8, "v0_rc4": 9.7, "v1_rc1": 9.6, "v1_rc2": 9.9,
+            "v1_rc4": 9.9}
+    assert P.corun_flags(base) == 0                       # best at once (9.6) gains < 5%: one after the other
+    t = dict(base, v1_rc2=8.0)
+    assert P.corun_flags(t) == 0b0111                     # at once, CD-2 kernel, op at GPU/2
+    t = dict(base, v0_rc4=7.0, v1_rc2=7.0)
+    assert P.corun_flags(t) == 0b0111                     # ties: the smaller flag word
+    t = dict(base, v0_rc4=6.0)
+    assert P.corun_flags(t) == 0b1001
+    # every configuration the table can record round-trips through the planner
+    import random as _r
+    from oracle import planner_ref as pr
+    for name, flags in P.CORUN_CONFIGS:
+        lut = P.write_lut([((7, 10, 12, 0), 4, [10, 11, 12, 13, 14], flags)], 132, 152)
+        conc, v, rc = pr.corun_plan(pr.Desc(128, 1024, 4096, 0), lut, pr.POLICY_AUTO)
+        assert conc == 1 and v == (11 if name.startswith("v1") else 10) and rc == int(name.split("rc")[1])

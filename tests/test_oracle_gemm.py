@@ -197,3 +197,23 @@ def test_workload_is_seeded():
     assert not np.array_equal(s1.a_bits(0), s1.a_bits(1))
     v = s1.a[0].to(torch.float32)
     assert float(v.min()) >= -1.0 and float(v.max()) <= 1.0
+
+
+def test_batched_gemm_is_block_diagonal_gemm():
+    """A batch of two GEMMs equals one GEMM of the concatenated A panels with
+    a block-diagonal B: [A0 A1] [[B0, 0], [0, B1]] = [A0 B0, A1 B1]."""
+    rng = np.random.default_rng(31)
+    M, K, N = 9, 70, 13
+    a = rng.integers(0, 65536, size=(2, M, K), dtype=np.uint32).astype(np.uint16)
+    a &= np.uint16(0xBFFF)        # finite values only (exponent below all-ones)
+    b = rng.integers(0, 65536, size=(2, K, N), dtype=np.uint32).astype(np.uint16)
+    b &= np.uint16(0xBFFF)
+    big_a = np.concatenate([a[0], a[1]], axis=1)
+    big_b = np.zeros((2 * K, 2 * N), dtype=np.uint16)          # bf16 +0
+    big_b[:K, :N] = b[0]
+    big_b[K:, N:] = b[1]
+    whole = og.gemm(big_a, big_b)
+    got = og.gemm_batched(a, b)
+    assert np.array_equal(got[0], whole[:, :N])
+    assert np.array_equal(got[1], whole[:, N:])
+    assert np.array_equal(og.gemm_batched(a[:1], b[:1])[0], og.gemm(a[0], b[0]))

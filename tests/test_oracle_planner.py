@@ -163,3 +163,35 @@ def test_preferred_cd_rule():
     assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.20, 8: 1.15}) == 4
     assert pr.preferred_cd({1: 1.0, 2: 0.8, 16: 1.9}) == 16
     assert pr.preferred_cd({1: 1.0}) == 1
+
+
+def test_corun_rule_by_hand():
+    # flags: bit 0 at once, bit 1 CD-2 kernel, bits 2-3 the op's cap index
+    e_go = pr.Entry((7, 10, 12, 0), 4, (10, 11, 12, 13, 14), 0b0111)     # at once, CD-2 kernel, op GPU/2
+    e_iso = pr.Entry((8, 10, 12, 0), 4, (30, 31, 32, 33, 34), 0b1001)    # at once, CD-1 kernel, op GPU/4
+    e_off = pr.Entry((9, 10, 12, 0), 1, (20, 21, 22, 23, 24), 0)
+    lut = pr.write_lut([e_go, e_iso, e_off], 132)
+    d_go, d_iso, d_off = pr.Desc(128, 1024, 4096, 0), pr.Desc(256, 1024, 4096, 0), pr.Desc(512, 1024, 4096, 0)
+    assert pr.corun_plan(d_go, lut, pr.POLICY_AUTO) == (1, 11, 2)
+    assert pr.corun_plan(d_iso, lut, pr.POLICY_AUTO) == (1, 30, 4)
+    assert pr.corun_plan(d_off, lut, pr.POLICY_AUTO) == (0, 20, 1)
+    for d, e in ((d_go, e_go), (d_off, e_off)):
+        assert pr.corun_plan(d, lut, pr.POLICY_SEQUENTIAL) == (0, e.variants[0], 1)
+        assert pr.corun_plan(d, lut, pr.POLICY_DEFAULT) == (1, e.variants[0], 1)
+        assert pr.corun_plan(d, lut, pr.POLICY_GO) == (1, e.variants[1], 2)
+    with pytest.raises(pr.PlanError):
+        pr.corun_plan(d_go, lut, pr.POLICY_FORCE_CD)
+    # a batched GEMM is bucketed by M * batch rows
+    assert pr.corun_plan(pr.Desc(64, 1024, 4096, 0, 2), lut, pr.POLICY_AUTO) == (1, 11, 2)
+
+
+def test_lut_flag_bits_round_trip_and_validation():
+    e = pr.Entry((7, 10, 12, 0), 4, (10, 11, 12, 13, 14), 0b1011)
+    data = pr.write_lut([e], 132)
+    assert data[32 + 5] == 0b1011
+    assert pr.parse_lut(data)[0][0].flags == 0b1011
+    for bad_flags in (0x10, 0b1100, 0x80):
+        bad = bytearray(data)
+        bad[32 + 5] = bad_flags
+        with pytest.raises(pr.LutError):
+            pr.parse_lut(bytes(bad))
