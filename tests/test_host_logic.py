@@ -86,12 +86,16 @@ def test_multi_rank_max_over_gloo():
 def test_corun_flags_rule():
     base = {"sequential": 10.0, "v0_rc1": 9.9, "v0_rc2": 9.8, "v0_rc4": 9.7, "v1_rc1": 9.6, "v1_rc2": 9.9,
             "v1_rc4": 9.9}
-    assert P.corun_flags(base) == 0                       # best at once (9.6) gains < 5%: one after the other
-    t = dict(base, v1_rc2=8.0)
-    assert P.corun_flags(t) == 0b0111                     # at once, CD-2 kernel, op at GPU/2
-    t = dict(base, v0_rc4=7.0, v1_rc2=7.0)
+    assert P.corun_flags(base) == 0                       # nothing at once gains 5% over one after the other
+    t = dict(base, v0_rc1=9.0)
+    assert P.corun_flags(t) == 0b0001                     # the default configuration at once
+    t = dict(base, v0_rc1=9.0, v1_rc2=8.8)
+    assert P.corun_flags(t) == 0b0001                     # 8.8 is not 5% better than the default's 9.0
+    t = dict(base, v0_rc1=9.0, v1_rc2=8.0)
+    assert P.corun_flags(t) == 0b0111                     # CD-2 kernel, op at GPU/2
+    t = dict(base, v0_rc1=9.0, v0_rc4=7.0, v1_rc2=7.0)
     assert P.corun_flags(t) == 0b0111                     # ties: the smaller flag word
-    t = dict(base, v0_rc4=6.0)
+    t = dict(base, v0_rc1=12.0, v0_rc4=9.0)
     assert P.corun_flags(t) == 0b1001
     # every configuration the table can record round-trips through the planner
     import random as _r
