@@ -58,6 +58,8 @@ def parse_args(argv=None):
                     help="fused: a wave's same-kind GEMMs share one launch; streams: one launch per GEMM")
     ap.add_argument("--replay", choices=["exec", "graph"], default="exec",
                     help="how the prepared step is replayed: recorded plain launches or a CUDA graph")
+    ap.add_argument("--serial-launch", action="store_true",
+                    help="plain serialised launches (no overlap of a launch's set-up with the previous kernel)")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--batched-study", default=None, metavar="FILE",
@@ -288,7 +290,7 @@ class SetRunner:
     once: a recorded prepared run (``replay="exec"``, plain launches) or a
     captured CUDA graph (``replay="graph"``)."""
 
-    def __init__(self, st, sched, copies, with_events=False, replay="exec"):
+    def __init__(self, st, sched, copies, with_events=False, replay="exec", serial_launch=False):
         import torch
         from paper_2409_02227_gb300 import goldy as G
         self.G = G
@@ -325,12 +327,11 @@ class SetRunner:
                 evs = {"ev_begin": [e.cuda_event for e in eb], "ev_end": [e.cuda_event for e in ee]}
                 self.events.append((eb, ee))
             if replay == "exec":
-                r = G.goldy_exec_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp, **evs)
-            elif evs:
-                r = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp,
-                                            evs["ev_begin"], evs["ev_end"])
+                r = G.goldy_exec_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp, serial_launch=serial_launch,
+                                        **evs)
             else:
-                r = G.goldy_graph_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp)
+                r = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp,
+                                            evs.get("ev_begin"), evs.get("ev_end"), serial_launch=serial_launch)
             self.runs.append(r)
         self.main = self.streams[0]
 
@@ -393,39 +394,37 @@ def time_schedule(st, sched, copies, steps, warm=10):
 
 
 def cublas_reference_ms(st, copies, steps):
-    """torch.matmul (cuBLAS) for the same set, back to back on one stream,
-    captured in a CUDA graph per rotating copy: a reference point only."""
+    """torch.matmul (cuBLAS) for the same set, back to back on one stream: one
+    CUDA graph runs the set once per rotating copy (so the inputs come from
+    HBM), replayed; ms per set.  A reference point only."""
     import torch
     base_a = [a.cuda() for a in st.a]
     base_b = [b.cuda() for b in st.b]
-    graphs = []
-    outs = []
-    keep = []                   # every captured graph reads its own inputs: keep them all alive
     s = torch.cuda.Stream()
+    keep = []                   # the captured graph reads every copy: keep them all alive
     for r in range(copies):
         A = base_a if r == 0 else [a.clone() for a in base_a]
         B = base_b if r == 0 else [b.clone() for b in base_b]
         keep.append((A, B))
-        with torch.cuda.stream(s):
-            for a, b in zip(A, B):
-                torch.matmul(a, b)          # warm cuBLAS handles outside the capture
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=s):
-            o = [torch.matmul(a, b) for a, b in zip(A, B)]
-        graphs.append(g)
-        outs.append(o)
-    for k in range(10):
-        graphs[k % copies].replay()
+    with torch.cuda.stream(s):
+        for a, b in zip(*keep[0]):
+            torch.matmul(a, b)      # warm cuBLAS handles outside the capture
     torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        outs = [[torch.matmul(a, b) for a, b in zip(A, B)] for A, B in keep]
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    reps = max(3, steps // copies)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    for k in range(steps):
-        graphs[k % copies].replay()
+    for _ in range(reps):
+        g.replay()
     e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / steps
-    del graphs, outs, keep
+    ms = e0.elapsed_time(e1) / (reps * copies)
+    del g, outs, keep
     return ms
 
 
@@ -496,7 +495,7 @@ def run_gpu(args, world, rank, local):
     in_bytes = sum(s.batch * (2 * s.M * s.K + 2 * s.K * s.N) for s in st.specs)
     copies = max(2, math.ceil(2 * l2 / in_bytes))
 
-    runner = SetRunner(st, sched, copies, replay=args.replay)
+    runner = SetRunner(st, sched, copies, replay=args.replay, serial_launch=args.serial_launch)
     for k in range(max(3, args.warmup)):
         runner.launch(k)
     torch.cuda.synchronize()
@@ -537,7 +536,7 @@ def run_gpu(args, world, rank, local):
         timing_note = (f"timed-region events / steps (one launch per step); events around each of the last "
                        f"{len(step_ms)} steps alone: {statistics.mean(step_ms) * 1e3:.2f} us")
     else:
-        inst = SetRunner(st, sched, copies, with_events=True, replay=args.replay)
+        inst = SetRunner(st, sched, copies, with_events=True, replay=args.replay, serial_launch=args.serial_launch)
         for k in range(2 * copies):
             inst.launch(k)
         torch.cuda.synchronize()
@@ -575,7 +574,8 @@ def run_gpu(args, world, rank, local):
                    "l2": f"inputs larger than L2: {copies} rotating device copies of the set "
                          f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2)",
                    "launch": f"{'prepared-run' if args.replay == 'exec' else 'CUDA graph'} replay of the planned "
-                             f"schedule ({args.launch} launch mode)",
+                             f"schedule ({args.launch} launch mode, "
+                             f"{'serialised launches' if args.serial_launch else 'each launch set-up overlapping the previous kernel (programmatic dependent launch)'})",
                    "plan": [{"gemm": i, "group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl,
                              "cd": cd} for i, (g, v, sl, cd) in enumerate(plan)],
                    "parallelism": f"replicas x{world}"},

@@ -282,6 +282,12 @@ typedef struct goldy_run_opts {
    * Null: no tracing. */
   void* trace;
   size_t trace_ctas;
+  /* 0 (default): each GO-Kernel launch may begin its set-up (barriers, tensor
+   * memory, descriptor prefetch) while the previous kernel on its stream is
+   * still running — programmatic dependent launch; the kernel waits for that
+   * kernel to complete before it touches global memory, so results and
+   * stream order are unchanged.  1: plain serialised launches. */
+  int32_t serial_launch;
 } goldy_run_opts;
 
 /* goldy_run with options; opts may be null (then identical to goldy_run). */

@@ -441,6 +441,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   unsigned long long* const trace = p.trace;
+  // the next launch on this stream may start its set-up now; it waits
+  // (griddep_wait) for this grid to complete before touching global memory
+  ptx::griddep_launch_dependents();
 
   if (threadIdx.x == 0) {
     trace_stamp(trace, kTrStart);
@@ -484,6 +487,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // have initialised them before any signal is sent
   if (p.cluster > 0) ptx::cluster_sync_all();
   const uint32_t tmem_base = *tmem_slot;
+  // set-up above touched only shared and tensor memory; global memory (the
+  // operands, C, the split-K workspace) only after the previous grid is done
+  ptx::griddep_wait();
   if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
   if (warp == 0) {

@@ -58,6 +58,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   const int pair = blockIdx.x >> 1;
   const int n_pairs = gridDim.x >> 1;
   unsigned long long* const trace = p.trace;
+  ptx::griddep_launch_dependents();   // see go_gemm_kernel
 
   if (threadIdx.x == 0) {
     trace_stamp(trace, kTrStart);
@@ -94,6 +95,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   ptx::cluster_sync_all();                  // the peer's barriers and tensor memory are ready
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  ptx::griddep_wait();                      // global memory only after the previous grid is done
   if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
   if (warp == 0) {

@@ -58,6 +58,7 @@ struct Op {
   unsigned block = 0;
   size_t smem = 0;
   int cluster = 0;
+  bool pdl = false;                  // programmatic dependency on the previous kernel of the stream
   std::vector<uint64_t> params;      // 8-byte-aligned copy of the parameter block
   void* ptr = nullptr;
   size_t pitch = 0, width = 0, height = 0;
@@ -66,6 +67,10 @@ struct Op {
 
 namespace {
 thread_local std::vector<Op>* t_rec = nullptr;   // non-null: record instead of enqueue
+// GO-Kernel launches carry a programmatic dependency on the previous kernel of
+// their stream (the kernels wait for it before touching global memory) unless
+// the run asks for serial launches
+thread_local bool t_pdl = true;
 }
 
 namespace {
@@ -159,27 +164,37 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
 // Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
 // cluster > 1.
 cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params,
-                              int cluster, unsigned block = kThreads) {
+                              int cluster, unsigned block = kThreads, bool pdl = false) {
   void* args[] = {params};
-  if (cluster <= 1) return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
+  if (cluster <= 1 && !pdl) return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(block);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = unsigned(cluster);
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  if (cluster > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = unsigned(cluster);
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  if (pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = n;
   return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
+// A GO-Kernel launch (recorded when t_rec is set).
 cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, const void* params,
                           size_t params_size, int cluster) {
-  if (!t_rec) return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster);
+  if (!t_rec) return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster, kThreads, t_pdl);
   Op op;
   op.kind = Op::kKernel;
   op.stream = stream;
@@ -187,6 +202,7 @@ cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream
   op.grid = grid;
   op.smem = smem;
   op.cluster = cluster;
+  op.pdl = t_pdl;
   op.params.resize((params_size + 7) / 8);
   std::memcpy(op.params.data(), params, params_size);
   t_rec->push_back(std::move(op));
@@ -253,7 +269,7 @@ cudaError_t replay(const Op& op) {
   switch (op.kind) {
     case Op::kKernel:
       return launch_kernel_now(op.fn, op.grid, op.smem, op.stream, const_cast<uint64_t*>(op.params.data()),
-                               op.cluster, op.block ? op.block : kThreads);
+                               op.cluster, op.block ? op.block : kThreads, op.pdl);
     case Op::kMemset2D: return cudaMemset2DAsync(op.ptr, op.pitch, 0, op.width, op.height, op.stream);
     case Op::kEventRecord: return cudaEventRecord(op.ev, op.stream);
     case Op::kEventRecordExternal: return cudaEventRecordWithFlags(op.ev, op.stream, 0);
@@ -666,6 +682,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
 
   t_trace = opts ? static_cast<unsigned long long*>(opts->trace) : nullptr;
   t_trace_ctas = opts ? opts->trace_ctas : 0;
+  t_pdl = !(opts && opts->serial_launch);
   auto hook = [&](void* const* evs, const int* members, int n, cudaStream_t stream) -> goldy_status {
     if (!evs) return GOLDY_OK;
     for (int j = 0; j < n; ++j) {
@@ -774,6 +791,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
   }
   t_trace = nullptr;
   t_trace_ctas = 0;
+  t_pdl = true;
   return ok();
 }
 

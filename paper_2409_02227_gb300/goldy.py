@@ -67,7 +67,7 @@ class goldy_gemm_desc(ctypes.Structure):
 
 class goldy_run_opts(ctypes.Structure):
     _fields_ = [("ev_begin", ctypes.POINTER(ctypes.c_void_p)), ("ev_end", ctypes.POINTER(ctypes.c_void_p)),
-                ("trace", ctypes.c_void_p), ("trace_ctas", ctypes.c_size_t)]
+                ("trace", ctypes.c_void_p), ("trace_ctas", ctypes.c_size_t), ("serial_launch", ctypes.c_int32)]
 
 
 class goldy_variant_info(ctypes.Structure):
@@ -360,10 +360,11 @@ def goldy_graph_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Seque
 
 
 def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]], trace: int = 0,
-          trace_ctas: int = 0):
+          trace_ctas: int = 0, serial_launch: bool = False):
     o = goldy_run_opts()
     o.trace = int(trace) or None
     o.trace_ctas = int(trace_ctas)
+    o.serial_launch = 1 if serial_launch else 0
     keep = []
     if ev_begin is not None:
         arr = _ptrs(ev_begin)
@@ -378,10 +379,12 @@ def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]], tr
 
 def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
                  workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
-                 ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0) -> None:
-    """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints)
-    and an optional device phase-trace buffer (see goldy_run_opts)."""
-    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas)
+                 ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0,
+                 serial_launch: bool = False) -> None:
+    """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints),
+    an optional device phase-trace buffer and the launch mode (see
+    goldy_run_opts)."""
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch)
     _check(_lib.goldy_run_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                              int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o)),
            "goldy_run_ex")
@@ -390,8 +393,8 @@ def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[in
 def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int],
                           workspace: int, workspace_bytes: int, streams: Sequence[int],
                           ev_begin: Optional[Sequence[int]] = None,
-                          ev_end: Optional[Sequence[int]] = None) -> Graph:
-    o, _keep = _opts(ev_begin, ev_end)
+                          ev_end: Optional[Sequence[int]] = None, serial_launch: bool = False) -> Graph:
+    o, _keep = _opts(ev_begin, ev_end, serial_launch=serial_launch)
     out = ctypes.c_void_p()
     _check(_lib.goldy_graph_create_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                                       int(workspace_bytes), _ptrs(streams), len(streams),
@@ -401,8 +404,9 @@ def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Se
 
 def goldy_exec_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
                       workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
-                      ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0) -> Exec:
-    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas)
+                      ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0,
+                      serial_launch: bool = False) -> Exec:
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch)
     out = ctypes.c_void_p()
     _check(_lib.goldy_exec_create(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                                   int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o),

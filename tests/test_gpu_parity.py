@@ -339,3 +339,40 @@ def test_sweep_sets_through_the_predictor_plan(cuda_ok, j):
     for i, s in enumerate(st.specs):
         rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(6, s.M))]))
         check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} (predictor plan) gemm {i} {s.M}x{s.N}x{s.K}")
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_dependent_launches_see_the_previous_kernels_output(cuda_ok, fused):
+    """Kernels of one stream overlap their set-up with the previous kernel
+    (programmatic dependent launch) but must read its results: a chain of
+    GEMMs, each reading the previous one's bf16 output as its A, run one after
+    another on one stream, matches the oracle chain, bit-identical to plain
+    serialised launches."""
+    M, N, K = 256, 512, 512
+    a0 = wl.random_matrix(M, K, 77, "normal", 0.05)
+    bs = [wl.random_matrix(K, N, 78 + j, "normal", 0.05) for j in range(4)]
+    descs = [G.desc(M, N, K, BF16)] * 4
+    vs = [vid(2, 1, 1), vid(3, 2, 2), vid(10, 1, 1), vid(2, 4, 4)]
+    s = G.goldy_schedule_build(descs, [0, 1, 2, 3], vs, [0, 0, 0, 0], G.GOLDY_PLAN_FUSED if fused else 0)
+    _, _, ms, ws_bytes = G.goldy_schedule_query(s)
+    ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+    dA0 = a0.cuda()
+    dB = [b.cuda() for b in bs]
+    outs = {}
+    for serial in (False, True):
+        dC = [torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(4)]
+        A = [dA0.data_ptr()] + [c.data_ptr() for c in dC[:3]]     # GEMM j reads GEMM j-1's output
+        st = torch.cuda.Stream()
+        st.wait_stream(torch.cuda.current_stream())
+        for _ in range(3):
+            G.goldy_run_ex(s, A, [b.data_ptr() for b in dB], [c.data_ptr() for c in dC], ws.data_ptr(), ws_bytes,
+                           [st.cuda_stream], serial_launch=serial)
+        torch.cuda.current_stream().wait_stream(st)
+        torch.cuda.synchronize()
+        assert G.goldy_device_error(clear=True) == 0
+        outs[serial] = [c.cpu() for c in dC]
+    prev = a0
+    for j in range(4):
+        check_close(outs[False][j], prev, bs[j], f"chain step {j}")
+        prev = outs[False][j]
+        assert torch.equal(outs[False][j].view(torch.int16), outs[True][j].view(torch.int16))
