@@ -354,15 +354,26 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
   }
 }
 
-// Cluster split-K with the partial tiles in shared memory: as reduce_slice,
-// but partial s is read from the shared memory of cluster CTA s (same
-// [chunk][float4][row] layout at `part_smem` in every CTA).
+// Shared-memory layout of a whole fp32 partial tile for the on-chip cluster
+// reduction: row-major, MMA_N / 4 granules of 16 bytes per row, granule f of
+// row r stored at position f ^ (r & 7) — a thread writing its accumulator row
+// and a warp reading consecutive granules of one row both hit distinct banks.
+template <int MMA_N>
+__device__ __forceinline__ uint32_t part_offset(int r, int f) {
+  return uint32_t(r * (MMA_N / 4) + (f ^ (r & 7))) * 16u;
+}
+
+// Cluster split-K with the partial tiles in shared memory: this CTA (split
+// `rank` of S) sums rows rank*128/S .. (rank+1)*128/S - 1 of the tile over
+// the S partials, partial s read from the shared memory of cluster CTA s, in
+// split order 0, 1, ..., S-1.  Consecutive threads take consecutive 16-byte
+// granules of a row, so C is written in whole rows.
 template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
 __device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part_smem, int rank, int m0, int n0,
                                                    int t) {
   constexpr int R = 128 / S;
-  constexpr int COLS4 = MMA_N / 4;
-  constexpr int PER_THREAD = R * COLS4 / 128;
+  constexpr int G4 = MMA_N / 4;                 // granules per row
+  constexpr int PER_THREAD = R * G4 / 128;
   constexpr int IB = (16 / S < PER_THREAD) ? 16 / S : PER_THREAD;
   static_assert(PER_THREAD >= 1 && PER_THREAD % IB == 0, "reduce tiling");
   const int r0 = rank * R;
@@ -375,7 +386,7 @@ __device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part
 #pragma unroll
     for (int b = 0; b < IB; ++b) {
       const int i = t + 128 * (k0 + b);
-      const uint32_t off = uint32_t((i / R) * 128 + r0 + (i % R)) * 16u;
+      const uint32_t off = part_offset<MMA_N>(r0 + i / G4, i % G4);
 #pragma unroll
       for (int s2 = 0; s2 < S; ++s2) vals[b][s2] = ptx::ld_shared_cluster_v4(peer[s2] + off);
     }
@@ -390,7 +401,7 @@ __device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part
         a.z += vals[b][s2].z;
         a.w += vals[b][s2].w;
       }
-      store_quad<SWAP, OUT_BF16>(w, m0, n0, r0 + (i % R), 4 * (i / R), a);
+      store_quad<SWAP, OUT_BF16>(w, m0, n0, r0 + i / G4, 4 * (i % G4), a);
     }
   }
 }
@@ -654,8 +665,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           ptx::tmem_ld_wait();
 #pragma unroll
           for (int j4 = 0; j4 < 8; ++j4)
-            ptx::st_shared_v4(part_smem + uint32_t(((c0 / 4) + j4) * 128 + r) * 16u, raw[4 * j4],
-                              raw[4 * j4 + 1], raw[4 * j4 + 2], raw[4 * j4 + 3]);
+            ptx::st_shared_v4(part_smem + part_offset<MMA_N>(r, c0 / 4 + j4), raw[4 * j4], raw[4 * j4 + 1],
+                              raw[4 * j4 + 2], raw[4 * j4 + 3]);
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
