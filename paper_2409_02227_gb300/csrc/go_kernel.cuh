@@ -102,6 +102,8 @@ enum : int {
   kTrArrived = 7,      // split-K: arrival counter bumped
   kTrFirstStore = 8,   // epilogue finished its first unit
   kTrEnd = 9,          // all roles done
+  kTrPreWait = 10,     // set-up done, about to wait for the grid this launch depends on
+  kTrProducerGo = 11,  // producer starts its first unit
   kTrUnits = 14,       // units processed by this CTA
   kTrSm = 15,          // SM id
   kTracePerCta = 16,
@@ -406,6 +408,54 @@ __device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part
   }
 }
 
+// Cluster split-K with pushed partials: CTA s of the S splits of a tile owns
+// rows s*128/S .. (s+1)*128/S - 1.  Every CTA sends the rows it does not own
+// to their owner (a bulk copy into the owner's receive slot, counted on the
+// owner's mbarrier) and keeps its own rows in its ring; the owner then sums,
+// from its own shared memory, the S partials of its rows in split order
+// 0, 1, ..., S-1 and stores them.  A slot holds 128/S rows in the layout of
+// part_offset; sender s goes to slot s (s < owner) or s - 1 (s > owner).
+template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
+__device__ __forceinline__ void reduce_slice_pushed(const CView& w, uint32_t own_slot, uint32_t recv_slots, int rank,
+                                                    int m0, int n0, int t) {
+  constexpr int R = 128 / S;
+  constexpr int G4 = MMA_N / 4;
+  constexpr int PER_THREAD = R * G4 / 128;
+  constexpr uint32_t SLOT_BYTES = uint32_t(R * MMA_N * 4);
+  static_assert(PER_THREAD >= 1 && (R * G4) % 128 == 0, "reduce tiling");
+  uint32_t src[S];
+#pragma unroll
+  for (int s2 = 0; s2 < S; ++s2)
+    src[s2] = s2 == rank ? own_slot : recv_slots + uint32_t(s2 < rank ? s2 : s2 - 1) * SLOT_BYTES;
+#pragma unroll 2
+  for (int k = 0; k < PER_THREAD; ++k) {
+    const int i = t + 128 * k;
+    const uint32_t off = part_offset<MMA_N>(i / G4, i % G4);
+    float4 v[S];
+#pragma unroll
+    for (int s2 = 0; s2 < S; ++s2) v[s2] = ptx::ld_shared_v4(src[s2] + off);
+    float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+    for (int s2 = 0; s2 < S; ++s2) {
+      a.x += v[s2].x;
+      a.y += v[s2].y;
+      a.z += v[s2].z;
+      a.w += v[s2].w;
+    }
+    store_quad<SWAP, OUT_BF16>(w, m0, n0, rank * R + i / G4, 4 * (i % G4), a);
+  }
+}
+
+// Bytes of the receive slots of the pushed reduction: the largest split
+// (8) leaves 7/8 of a 128 x MMA_N fp32 tile to receive.  Kinds that own a
+// whole SM with MMA_N <= 128 have room for them (the host's shared-memory
+// size per kind reserves the same bytes).
+template <int MMA_N, int MIN_CTAS>
+struct PushRecv {
+  static constexpr bool enabled = MIN_CTAS == 1 && MMA_N <= 128;
+  static constexpr int bytes = enabled ? 7 * 128 * MMA_N * 4 / 8 : 0;
+};
+
 template <int MMA_N, int ACC>
 struct TmemCols {
   static constexpr uint32_t need = uint32_t(MMA_N * ACC);
@@ -434,17 +484,24 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   constexpr int STAGING_BYTES = EPI_TMA ? 2 * 16384 : 0;
   // a whole fp32 partial tile fits in the ring's shared memory
   constexpr bool kPartFitsRing = STAGES * STAGE_BYTES >= 128 * MMA_N * 4;
+  // pushed cluster reduction: receive slots share the region after the ring
+  // with the TMA-store staging buffers (a launch uses one or the other: the
+  // pushed reduction runs only when every GEMM of the launch is split)
+  constexpr bool kPush = PushRecv<MMA_N, MIN_CTAS>::enabled;
+  constexpr int EPI_BYTES =
+      STAGING_BYTES > PushRecv<MMA_N, MIN_CTAS>::bytes ? STAGING_BYTES : PushRecv<MMA_N, MIN_CTAS>::bytes;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + STAGING_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + EPI_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* tfull = bars + 2 * STAGES;
   uint64_t* tempty = bars + 2 * STAGES + ACC;
   uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
   uint64_t* redbar = drain + 1;        // cluster split-K: 2 barriers, alternating by unit
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(redbar + 2);
+  uint64_t* recvbar = redbar + 2;      // pushed cluster reduction: bytes received
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
 
@@ -455,6 +512,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // the next launch on this stream may start its set-up now; it waits
   // (griddep_wait) for this grid to complete before touching global memory
   ptx::griddep_launch_dependents();
+
+  // pushed cluster reduction: one unit per CTA, every GEMM split S = cluster
+  const bool push_on = kPush && p.cluster > 0 && p.total_units == int(gridDim.x);
 
   if (threadIdx.x == 0) {
     trace_stamp(trace, kTrStart);
@@ -482,10 +542,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       ptx::mbar_init(ptx::smem_u32(&redbar[0]), uint32_t(p.cluster));
       ptx::mbar_init(ptx::smem_u32(&redbar[1]), uint32_t(p.cluster));
     }
+    if (push_on) ptx::mbar_init(ptx::smem_u32(recvbar), 1);
     *abort_flag = 0;
     *last_flag = 0;
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
+    // the phase completes once the S - 1 peers' rows of this CTA's slice
+    // have landed (peers start sending only after the cluster-wide sync below)
+    if (push_on)
+      ptx::mbar_arrive_expect_tx(ptx::smem_u32(recvbar),
+                                 uint32_t((p.cluster - 1) * (128 / p.cluster) * MMA_N * 4));
   }
   if (warp == 1) {
     ptx::tmem_alloc(ptx::smem_u32(tmem_slot), TMEM_COLS);
@@ -498,6 +564,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // have initialised them before any signal is sent
   if (p.cluster > 0) ptx::cluster_sync_all();
   const uint32_t tmem_base = *tmem_slot;
+  if (threadIdx.x == 0) trace_stamp(trace, kTrPreWait);
   // set-up above touched only shared and tensor memory; global memory (the
   // operands, C, the split-K workspace) only after the previous grid is done
   ptx::griddep_wait();
@@ -510,6 +577,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       uint32_t phase = 0, issued = 0, last_phase = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
+        if (issued == 0) trace_stamp(trace, kTrProducerGo);
         const UnitCoord c = decode_unit(p, u);
         const void* ta = &p.tmap_a[c.g];
         const void* tb = &p.tmap_b[c.g];
@@ -648,6 +716,59 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
           store_chunk<SWAP, OUT_BF16>(cv, m0, n0, r, c0, v);
+        }
+      } else if (push_on) {
+        // ---- cluster split-K, pushed: one unit per CTA.  Row r of the
+        // accumulator belongs to the CTA of rank r / (128/S).  The partial
+        // goes into the ring (free once the accumulator is complete) as S
+        // slices of 128/S rows; one bulk copy per peer sends it its slice,
+        // counted on the peer's receive barrier.  Then wait until every
+        // peer's copy of this CTA's slice has landed and reduce the S slices
+        // from local shared memory.  The cluster barrier at kernel exit keeps
+        // every source buffer alive until its copies have landed.
+        const int S = w.split;
+        const int R = 128 / S;
+        const int d = r / R;                   // rank that reduces this row
+        const int rr = r - d * R;              // row within that rank's slice
+        const uint32_t slot_bytes = uint32_t(R * MMA_N * 4);
+        const uint32_t stage_row = tiles_base + uint32_t(d) * slot_bytes;
+        const uint32_t recv_slots = tiles_base + uint32_t(STAGES * STAGE_BYTES);
+#pragma unroll 1
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int j4 = 0; j4 < 8; ++j4)
+            ptx::st_shared_v4(stage_row + part_offset<MMA_N>(rr, c0 / 4 + j4), raw[4 * j4], raw[4 * j4 + 1],
+                              raw[4 * j4 + 2], raw[4 * j4 + 3]);
+        }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
+        released = true;
+        ptx::fence_proxy_async_smem();                   // slices visible to the bulk copies
+        ptx::named_bar_sync(1, 128);
+        if (et < S && et != c.s) {
+          const uint32_t slot = uint32_t(c.s < et ? c.s : c.s - 1);
+          ptx::bulk_copy_to_peer(ptx::map_to_rank(recv_slots + slot * slot_bytes, uint32_t(et)),
+                                 tiles_base + uint32_t(et) * slot_bytes, slot_bytes,
+                                 ptx::map_to_rank(ptx::smem_u32(recvbar), uint32_t(et)));
+        }
+        if (first_unit && et == 0) trace_stamp(trace, kTrPartials);
+        bool ok2 = ptx::mbar_wait_cluster(ptx::smem_u32(recvbar), 0, abort_flag);
+        ok2 = ptx::named_bar_and(1, 128, ok2);
+        if (!ok2) {
+          if (et == 0) raise_error(p.err, abort_flag, kErrClusterWait);
+          break;
+        }
+        if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
+        const uint32_t own_slot = tiles_base + uint32_t(c.s) * slot_bytes;
+        switch (S) {
+          case 2: reduce_slice_pushed<MMA_N, 2, SWAP, OUT_BF16>(cv, own_slot, recv_slots, c.s, m0, n0, et); break;
+          case 4: reduce_slice_pushed<MMA_N, 4, SWAP, OUT_BF16>(cv, own_slot, recv_slots, c.s, m0, n0, et); break;
+          case 8: reduce_slice_pushed<MMA_N, 8, SWAP, OUT_BF16>(cv, own_slot, recv_slots, c.s, m0, n0, et); break;
+          default: break;
         }
       } else if (kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x)) {
         // ---- cluster split-K on chip: one unit per CTA, so the ring's shared

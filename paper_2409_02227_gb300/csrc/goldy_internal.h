@@ -45,7 +45,7 @@ inline constexpr KindInfo kKinds[kNumKinds] = {
     // name        mma_n swap stages acc ctas/SM pair
     {"n64_full", 64, 0, 8, 2, 1, 0},
     {"n64_half", 64, 0, 4, 2, 2, 0},
-    {"n128_full", 128, 0, 6, 2, 1, 0},
+    {"n128_full", 128, 0, 5, 2, 1, 0},
     {"n128_half", 128, 0, 3, 2, 2, 0},
     {"n256_full", 256, 0, 4, 2, 1, 0},
     {"n256_half", 256, 0, 2, 1, 2, 0},
@@ -69,9 +69,20 @@ constexpr int tmem_cols(const KindInfo& k) {
 // Kinds with a whole SM to themselves (and the pair kind) store C through
 // shared memory with TMA; they keep two 16 KB staging buffers.
 constexpr bool epi_tma(const KindInfo& k) { return k.pair || (!k.swap_ab && k.ctas_per_sm == 1); }
-// stages, staging, 1 KB for 1024-byte alignment of the swizzled tiles, 1 KB for barriers
+// Kinds with a whole SM to themselves and tiles at most 128 wide reduce
+// cluster split-K by pushing partial rows into receive slots of their peers:
+// up to 7/8 of a 128 x mma_n fp32 tile (split 8).  The slots share one region
+// with the TMA-store staging buffers (a launch uses one or the other).
+constexpr int push_recv_bytes(const KindInfo& k) {
+  return (!k.pair && k.ctas_per_sm == 1 && k.mma_n <= 128) ? 7 * kMmaM * k.mma_n * 4 / 8 : 0;
+}
+constexpr int epilogue_bytes(const KindInfo& k) {
+  return (epi_tma(k) ? 2 * 16384 : 0) > push_recv_bytes(k) ? (epi_tma(k) ? 2 * 16384 : 0) : push_recv_bytes(k);
+}
+// stages, epilogue region, 1 KB for 1024-byte alignment of the swizzled
+// tiles, 1 KB for barriers
 constexpr int smem_bytes(const KindInfo& k) {
-  return k.stages * stage_bytes(k) + (epi_tma(k) ? 2 * 16384 : 0) + 2048;
+  return k.stages * stage_bytes(k) + epilogue_bytes(k) + 2048;
 }
 
 struct Variant {

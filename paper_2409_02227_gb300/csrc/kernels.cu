@@ -20,6 +20,9 @@ template <int KIND>
 const void* select_kernel(int out_bf16, int fused) {
   constexpr KindInfo k = kKinds[KIND];
   constexpr bool swap = k.swap_ab != 0;
+  static_assert(k.pair != 0 || PushRecv<k.mma_n, k.ctas_per_sm>::bytes == push_recv_bytes(k),
+                "host and kernel agree on the pushed reduction's receive slots");
+  static_assert(smem_bytes(k) <= 232448, "shared memory per CTA");
   if constexpr (k.pair != 0) {
     if (fused)
       return out_bf16 ? reinterpret_cast<const void*>(&go_gemm_pair_kernel<true, kMaxFused>)

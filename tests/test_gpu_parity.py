@@ -42,7 +42,7 @@ def test_each_kind_ragged(cuda_ok, kind, out):
 
 
 @pytest.mark.parametrize("split", [2, 4, 8])
-@pytest.mark.parametrize("kind", [0, 3, 5, 6, 9])
+@pytest.mark.parametrize("kind", [0, 2, 3, 5, 6, 8, 9])
 def test_split_k(cuda_ok, kind, split):
     M, N, K = (48, 256, 1024) if kind in SWAP_KINDS else (130, 256, 1024)
     a, b = inputs(M, N, K, seed=100 + kind * 10 + split)
@@ -73,7 +73,7 @@ def test_k_tail_and_odd_m(cuda_ok, kind):
     check_close(c, a, b, f"kind {kind} K tail")
 
 
-@pytest.mark.parametrize("kind", [0, 3, 6])
+@pytest.mark.parametrize("kind", [0, 2, 3, 6, 8])
 def test_grid_cap_is_bit_exact(cuda_ok, kind):
     # the resource constraint changes how many CTAs share the units, never the math
     M, N, K = (64, 4096, 512) if kind in SWAP_KINDS else (512, 1024, 512)
