@@ -276,10 +276,13 @@ typedef struct goldy_run_opts {
    * (k: 0 entry, 1 set-up done, 2 first TMA load, 3 first full stage seen by
    * the MMA thread, 4 first accumulator committed, 5 first accumulator seen
    * by the epilogue, 6 split-K partial stored, 7 split-K arrival counted,
-   * 8 first unit stored, 9 exit — %globaltimer nanoseconds; 14 units this CTA
-   * processed; 15 SM id).  Size it for the largest grid (trace_ctas CTAs);
-   * launches of one run share it, so use it on single-launch schedules.
-   * Null: no tracing. */
+   * 8 first unit stored, 9 exit, 10 set-up done before waiting for the
+   * previous kernel on the stream, 11 producer started — %globaltimer
+   * nanoseconds; 12 the launch's grid size; 13 the CTA's index in its launch;
+   * 14 units this CTA processed; 15 SM id).  The launches of one run use
+   * consecutive regions in launch order (launch j starts after the CTAs of
+   * launches 0 .. j-1); a launch that does not fit in the trace_ctas CTAs
+   * left is not traced.  Null: no tracing. */
   void* trace;
   size_t trace_ctas;
   /* 0 (default): each GO-Kernel launch may begin its set-up (barriers, tensor

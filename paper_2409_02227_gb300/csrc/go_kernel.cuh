@@ -104,6 +104,8 @@ enum : int {
   kTrEnd = 9,          // all roles done
   kTrPreWait = 10,     // set-up done, about to wait for the grid this launch depends on
   kTrProducerGo = 11,  // producer starts its first unit
+  kTrGrid = 12,        // grid size of the launch (launches of one run trace into consecutive regions)
+  kTrCta = 13,         // CTA index within its launch
   kTrUnits = 14,       // units processed by this CTA
   kTrSm = 15,          // SM id
   kTracePerCta = 16,
@@ -528,6 +530,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       uint32_t sm;
       asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
       trace[blockIdx.x * kTracePerCta + kTrSm] = sm;
+      trace[blockIdx.x * kTracePerCta + kTrGrid] = gridDim.x;
+      trace[blockIdx.x * kTracePerCta + kTrCta] = blockIdx.x;
     }
     for (int s = 0; s < STAGES; ++s) {
       ptx::mbar_init(ptx::smem_u32(&full[s]), 1);

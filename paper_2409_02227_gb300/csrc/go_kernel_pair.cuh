@@ -66,6 +66,8 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       uint32_t sm;
       asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
       trace[blockIdx.x * kTracePerCta + kTrSm] = sm;
+      trace[blockIdx.x * kTracePerCta + kTrGrid] = gridDim.x;
+      trace[blockIdx.x * kTracePerCta + kTrCta] = blockIdx.x;
     }
     for (int g = 0; g < p.n_gemms; ++g) {
       ptx::prefetch_tensormap(&p.tmap_a[g]);

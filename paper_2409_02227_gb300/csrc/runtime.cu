@@ -47,6 +47,9 @@ void runtime_release(Runtime* rt) {
   delete rt;
 }
 
+// Launch priority value meaning "none": the launch takes its stream's priority.
+constexpr int kNoPriority = 1 << 30;
+
 // One enqueued operation of a run.  goldy_run_ex executes them as it goes;
 // goldy_exec_create records them (with copies of the kernel parameter blocks)
 // so goldy_exec_launch can replay the run with plain launch calls.
@@ -59,6 +62,7 @@ struct Op {
   size_t smem = 0;
   int cluster = 0;
   bool pdl = false;                  // programmatic dependency on the previous kernel of the stream
+  int prio = kNoPriority;            // launch priority (kNoPriority: the stream's)
   std::vector<uint64_t> params;      // 8-byte-aligned copy of the parameter block
   void* ptr = nullptr;
   size_t pitch = 0, width = 0, height = 0;
@@ -71,6 +75,10 @@ thread_local std::vector<Op>* t_rec = nullptr;   // non-null: record instead of 
 // their stream (the kernels wait for it before touching global memory) unless
 // the run asks for serial launches
 thread_local bool t_pdl = true;
+// Launch priority of the next GO-Kernel launch (kNoPriority: the stream's).
+// A heterogeneous fused wave ranks its launches by work so the block
+// scheduler hands SMs to the largest first and the others fill its tail.
+thread_local int t_prio = kNoPriority;
 }
 
 namespace {
@@ -80,6 +88,7 @@ constexpr int kMaxDevices = 64;
 struct DeviceState {
   bool init = false;
   int sm_count = 0;
+  int prio_least = 0, prio_greatest = 0;    // cudaDeviceGetStreamPriorityRange
   int* err_word = nullptr;
   int ctas_per_sm[kNumKinds][2][2] = {};   // [kind][bf16 out][fused]; 0 = not yet set up
   int cluster_ok[kNumKinds][2][2][4] = {};  // [..][log2 cluster size]; 0 unknown, 1 yes, -1 no
@@ -121,6 +130,8 @@ goldy_status device_state(DeviceState** out) {
   if (!d.init) {
     e = cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    e = cudaDeviceGetStreamPriorityRange(&d.prio_least, &d.prio_greatest);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetStreamPriorityRange");
     e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err_word), g_device_error);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
     if (!g_encode) {
@@ -164,16 +175,22 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
 // Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
 // cluster > 1.
 cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params,
-                              int cluster, unsigned block = kThreads, bool pdl = false) {
+                              int cluster, unsigned block = kThreads, bool pdl = false, int prio = kNoPriority) {
   void* args[] = {params};
-  if (cluster <= 1 && !pdl) return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
+  if (cluster <= 1 && !pdl && prio == kNoPriority)
+    return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(block);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[3];
   unsigned n = 0;
+  if (prio != kNoPriority) {
+    attr[n].id = cudaLaunchAttributePriority;
+    attr[n].val.priority = prio;
+    ++n;
+  }
   if (cluster > 1) {
     attr[n].id = cudaLaunchAttributeClusterDimension;
     attr[n].val.clusterDim.x = unsigned(cluster);
@@ -194,7 +211,8 @@ cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaSt
 // A GO-Kernel launch (recorded when t_rec is set).
 cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, const void* params,
                           size_t params_size, int cluster) {
-  if (!t_rec) return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster, kThreads, t_pdl);
+  if (!t_rec)
+    return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster, kThreads, t_pdl, t_prio);
   Op op;
   op.kind = Op::kKernel;
   op.stream = stream;
@@ -203,6 +221,7 @@ cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream
   op.smem = smem;
   op.cluster = cluster;
   op.pdl = t_pdl;
+  op.prio = t_prio;
   op.params.resize((params_size + 7) / 8);
   std::memcpy(op.params.data(), params, params_size);
   t_rec->push_back(std::move(op));
@@ -269,7 +288,7 @@ cudaError_t replay(const Op& op) {
   switch (op.kind) {
     case Op::kKernel:
       return launch_kernel_now(op.fn, op.grid, op.smem, op.stream, const_cast<uint64_t*>(op.params.data()),
-                               op.cluster, op.block ? op.block : kThreads, op.pdl);
+                               op.cluster, op.block ? op.block : kThreads, op.pdl, op.prio);
     case Op::kMemset2D: return cudaMemset2DAsync(op.ptr, op.pitch, 0, op.width, op.height, op.stream);
     case Op::kEventRecord: return cudaEventRecord(op.ev, op.stream);
     case Op::kEventRecordExternal: return cudaEventRecordWithFlags(op.ev, op.stream, 0);
@@ -404,7 +423,6 @@ goldy_status launch_degenerate(const GemmPlan& gp, void* C, cudaStream_t stream)
   return GOLDY_OK;
 }
 
-// Phase-trace buffer of the current goldy_run_ex call (null: off).
 // ---------------------------------------------------------------------------
 // SM partitions (CUDA green contexts).  A partition is a green context owning
 // a subset of the SMs; work on its streams runs on those SMs only.  Every
@@ -497,11 +515,18 @@ class PartitionScope {
 };
 int sms(const DeviceState& d) { return t_sms > 0 ? std::min(t_sms, d.sm_count) : d.sm_count; }
 
+// Phase-trace buffer of the current goldy_run_ex call (null: off).
 thread_local unsigned long long* t_trace = nullptr;
 thread_local size_t t_trace_ctas = 0;
+thread_local size_t t_trace_used = 0;   // CTAs of the run's earlier launches
 
+// The launches of one run trace into consecutive regions of the buffer, in
+// launch order; a launch that does not fit in what is left is not traced.
 unsigned long long* trace_for(unsigned grid) {
-  return (t_trace && grid <= t_trace_ctas) ? t_trace : nullptr;
+  if (!t_trace || t_trace_used + grid > t_trace_ctas) return nullptr;
+  unsigned long long* region = t_trace + t_trace_used * 16;
+  t_trace_used += grid;
+  return region;
 }
 
 // scale > 0: the launch's grid cap is its variant's cap times `scale` (set for
@@ -682,6 +707,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
 
   t_trace = opts ? static_cast<unsigned long long*>(opts->trace) : nullptr;
   t_trace_ctas = opts ? opts->trace_ctas : 0;
+  t_trace_used = 0;
   t_pdl = !(opts && opts->serial_launch);
   auto hook = [&](void* const* evs, const int* members, int n, cudaStream_t stream) -> goldy_status {
     if (!evs) return GOLDY_OK;
@@ -701,6 +727,8 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
     struct LaunchSet {
       int slot, n, degenerate, wave;
       double scale;     // grid-cap scale for heterogeneous fused waves (0: none)
+      int prio;         // launch priority (kNoPriority: the stream's)
+      double flops;
       int members[kMaxFused];
     };
     LaunchSet sets[GOLDY_MAX_GEMMS];
@@ -729,8 +757,12 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
           sets[target].degenerate = degenerate(gp) ? 1 : 0;
           sets[target].wave = w0;
           sets[target].scale = 0.0;
+          sets[target].prio = kNoPriority;
+          sets[target].flops = 0.0;
         }
         sets[target].members[sets[target].n++] = i;
+        sets[target].flops += 2.0 * double(gp.desc.M) * double(gp.desc.N) * double(gp.desc.K) *
+                              double(std::max<int64_t>(1, gp.desc.batch));
       }
     }
     // A fused wave whose GEMMs are of different kinds runs one launch per
@@ -748,8 +780,21 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
           ++t1;
         }
         if (kernels > 1)
-          for (int t = t0; t < t1; ++t)
-            if (!sets[t].degenerate) sets[t].scale = double(wave_size) / double(sets[t].n);
+          for (int t = t0; t < t1; ++t) {
+            if (sets[t].degenerate) continue;
+            sets[t].scale = double(wave_size) / double(sets[t].n);
+            // rank by work (ties: launch order); rank 0 gets the device's
+            // greatest priority, each further rank one step less
+            int rank = 0;
+            for (int u = t0; u < t1; ++u)
+              if (u != t && !sets[u].degenerate &&
+                  (sets[u].flops > sets[t].flops || (sets[u].flops == sets[t].flops && u < t)))
+                ++rank;
+            const int step = d->prio_greatest <= d->prio_least ? 1 : -1;
+            int pr = d->prio_greatest + step * rank;
+            if ((step > 0 && pr > d->prio_least) || (step < 0 && pr < d->prio_least)) pr = d->prio_least;
+            sets[t].prio = pr;
+          }
         t0 = t1;
       }
     }
@@ -770,12 +815,14 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
       cudaStream_t stream = static_cast<cudaStream_t>(streams[ls.slot]);
       st = hook(opts ? opts->ev_begin : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
+      t_prio = ls.prio;
       if (ls.n == 1) {
         const int i = ls.members[0];
         st = launch_gemm(*d, s->gemms[i], A[i], B[i], C[i], ws, stream, ls.scale);
       } else {
         st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream, ls.scale);
       }
+      t_prio = kNoPriority;
       if (st != GOLDY_OK) return st;
       st = hook(opts ? opts->ev_end : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
@@ -791,6 +838,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
   }
   t_trace = nullptr;
   t_trace_ctas = 0;
+  t_trace_used = 0;
   t_pdl = true;
   return ok();
 }
