@@ -719,30 +719,32 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
   };
   const bool fused = (s->flags & GOLDY_PLAN_FUSED) != 0;
 
-  for (const Group& grp : s->groups) {
-    // Launch sets.  Streams mode: one per GEMM, on the GEMM's slot.  Fused
-    // mode: the group's members taken CD at a time form waves; in a wave, the
-    // GEMMs of one kind and output dtype share a launch on the slot of the
-    // first of them.
-    struct LaunchSet {
-      int slot, n, degenerate, wave;
-      double scale;     // grid-cap scale for heterogeneous fused waves (0: none)
-      int prio;         // launch priority (kNoPriority: the stream's)
-      double flops;
-      int members[kMaxFused];
-    };
-    LaunchSet sets[GOLDY_MAX_GEMMS];
-    int n_sets = 0;
+  // Launch sets.  Streams mode: one per GEMM, on the GEMM's slot.  Fused
+  // mode: a group's members taken CD at a time form waves; in a wave, the
+  // GEMMs of one kind and output dtype share a launch on the slot of the
+  // first of them.
+  struct LaunchSet {
+    int group, slot, n, degenerate, wave;
+    double scale;     // grid-cap scale for heterogeneous fused waves (0: none)
+    int rank;         // rank by FLOPs among the launches of its wave (0: largest)
+    int prio;         // launch priority (kNoPriority: the stream's)
+    double flops;
+    int members[kMaxFused];
+  };
+  std::vector<LaunchSet> sets;
+  sets.reserve(s->gemms.size());
+  for (size_t g = 0; g < s->groups.size(); ++g) {
+    const Group& grp = s->groups[g];
     const int size = int(grp.members.size());
     const int wave = fused ? std::max(1, grp.cd) : 1;
     for (int w0 = 0; w0 < size; w0 += wave) {
-      const int first_set = n_sets;
+      const size_t first_set = sets.size();
       for (int j = w0; j < std::min(size, w0 + wave); ++j) {
         const int i = grp.members[j];
         const GemmPlan& gp = s->gemms[i];
-        int target = -1;
+        size_t target = sets.size();
         if (fused && !degenerate(gp))
-          for (int t = first_set; t < n_sets; ++t) {
+          for (size_t t = first_set; t < sets.size(); ++t) {
             const GemmPlan& g0 = s->gemms[sets[t].members[0]];
             if (!sets[t].degenerate && sets[t].n < kMaxFused && g0.kind == gp.kind &&
                 g0.desc.c_dtype == gp.desc.c_dtype) {
@@ -750,71 +752,104 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
               break;
             }
           }
-        if (target < 0) {
-          target = n_sets++;
-          sets[target].slot = gp.slot;
-          sets[target].n = 0;
-          sets[target].degenerate = degenerate(gp) ? 1 : 0;
-          sets[target].wave = w0;
-          sets[target].scale = 0.0;
-          sets[target].prio = kNoPriority;
-          sets[target].flops = 0.0;
+        if (target == sets.size()) {
+          LaunchSet ls{};
+          ls.group = int(g);
+          ls.slot = gp.slot;
+          ls.degenerate = degenerate(gp) ? 1 : 0;
+          ls.wave = w0;
+          ls.prio = kNoPriority;
+          sets.push_back(ls);
         }
         sets[target].members[sets[target].n++] = i;
         sets[target].flops += 2.0 * double(gp.desc.M) * double(gp.desc.N) * double(gp.desc.K) *
                               double(std::max<int64_t>(1, gp.desc.batch));
       }
     }
-    // A fused wave whose GEMMs are of different kinds runs one launch per
-    // kind, side by side.  A GO-Kernel tuned for CD c was sized as one of c
-    // co-runners sharing the GPU; a launch that carries m of the wave's c
-    // GEMMs therefore gets c/m times its members' caps (at most the whole
-    // GPU).  Launches go out largest first, so smaller ones fill the SMs the
-    // larger one frees in its tail.
-    if (fused) {
-      for (int t0 = 0; t0 < n_sets;) {
-        int t1 = t0, kernels = 0, wave_size = 0;
-        while (t1 < n_sets && sets[t1].wave == sets[t0].wave) {
-          wave_size += sets[t1].n;
-          if (!sets[t1].degenerate) ++kernels;
-          ++t1;
-        }
-        if (kernels > 1)
-          for (int t = t0; t < t1; ++t) {
-            if (sets[t].degenerate) continue;
-            sets[t].scale = double(wave_size) / double(sets[t].n);
-            // rank by work (ties: launch order); rank 0 gets the device's
-            // greatest priority, each further rank one step less
-            int rank = 0;
-            for (int u = t0; u < t1; ++u)
-              if (u != t && !sets[u].degenerate &&
-                  (sets[u].flops > sets[t].flops || (sets[u].flops == sets[t].flops && u < t)))
-                ++rank;
-            const int step = d->prio_greatest <= d->prio_least ? 1 : -1;
-            int pr = d->prio_greatest + step * rank;
-            if ((step > 0 && pr > d->prio_least) || (step < 0 && pr < d->prio_least)) pr = d->prio_least;
-            sets[t].prio = pr;
-          }
-        t0 = t1;
+  }
+  // Priority levels from the device's greatest (level 0) to its least.
+  const int prio_step = d->prio_greatest <= d->prio_least ? 1 : -1;
+  const int prio_levels = std::abs(d->prio_least - d->prio_greatest) + 1;
+  auto level = [&](int lv) { return d->prio_greatest + prio_step * std::min(lv, prio_levels - 1); };
+  // A fused wave whose GEMMs are of different kinds runs one launch per
+  // kind, side by side.  A GO-Kernel tuned for CD c was sized as one of c
+  // co-runners sharing the GPU; a launch that carries m of the wave's c GEMMs
+  // therefore gets c/m times its members' caps (at most the whole GPU), and
+  // the wave's launches are ranked by FLOPs into launch priorities, so the
+  // largest gets the SMs first and smaller ones fill the SMs it frees in its
+  // tail.
+  const bool soft_groups = fused && s->groups.size() > 1;
+  if (fused) {
+    for (size_t t0 = 0; t0 < sets.size();) {
+      size_t t1 = t0;
+      int kernels = 0, wave_size = 0;
+      while (t1 < sets.size() && sets[t1].group == sets[t0].group && sets[t1].wave == sets[t0].wave) {
+        wave_size += sets[t1].n;
+        if (!sets[t1].degenerate) ++kernels;
+        ++t1;
       }
-    }
-    uint32_t used = 0;
-    for (int t = 0; t < n_sets; ++t) used |= 1u << sets[t].slot;
-    const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
-    if (side) {
-      cudaError_t e = enq_event_record(rt->fork, main);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
-      for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
-        if (side >> k & 1) {
-          e = enq_wait(static_cast<cudaStream_t>(streams[k]), rt->fork);
-          if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+      for (size_t t = t0; t < t1; ++t) {
+        if (sets[t].degenerate) continue;
+        for (size_t u = t0; u < t1; ++u)
+          if (u != t && !sets[u].degenerate &&
+              (sets[u].flops > sets[t].flops || (sets[u].flops == sets[t].flops && u < t)))
+            ++sets[t].rank;
+        if (kernels > 1) {
+          sets[t].scale = double(wave_size) / double(sets[t].n);
+          sets[t].prio = level(sets[t].rank);
         }
+        // groups of a fused plan are not separated by a join: group g's
+        // launches rank g levels below the first group's, so a later group
+        // fills the SMs an earlier group frees in its tail
+        if (soft_groups) sets[t].prio = level(sets[t].group + sets[t].rank);
+      }
+      t0 = t1;
     }
-    for (int t = 0; t < n_sets; ++t) {
+  }
+  // Fork the side streams from streams[0] and join them back: around each
+  // group in streams mode (groups run one after another), once around the
+  // whole run in fused mode.
+  auto fork = [&](uint32_t side) -> goldy_status {
+    if (!side) return GOLDY_OK;
+    cudaError_t e = enq_event_record(rt->fork, main);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
+      if (side >> k & 1) {
+        e = enq_wait(static_cast<cudaStream_t>(streams[k]), rt->fork);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+      }
+    return GOLDY_OK;
+  };
+  auto join = [&](uint32_t side) -> goldy_status {
+    for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
+      if (side >> k & 1) {
+        cudaError_t e = enq_event_record(rt->join[k], static_cast<cudaStream_t>(streams[k]));
+        if (e == cudaSuccess) e = enq_wait(main, rt->join[k]);
+        if (e != cudaSuccess) return cuda_fail(e, "join event");
+      }
+    return GOLDY_OK;
+  };
+  const bool pdl = t_pdl;
+  int last_group[GOLDY_MAX_STREAMS];
+  for (int k = 0; k < GOLDY_MAX_STREAMS; ++k) last_group[k] = -1;
+  for (size_t t0 = 0; t0 < sets.size();) {
+    // the launches dispatched between one fork and its join
+    size_t t1 = t0;
+    while (t1 < sets.size() && (fused || sets[t1].group == sets[t0].group)) ++t1;
+    uint32_t used = 0;
+    for (size_t t = t0; t < t1; ++t) used |= 1u << sets[t].slot;
+    const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
+    st = fork(side);
+    if (st != GOLDY_OK) return st;
+    for (size_t t = t0; t < t1; ++t) {
       const LaunchSet& ls = sets[t];
       cudaStream_t stream = static_cast<cudaStream_t>(streams[ls.slot]);
       st = hook(opts ? opts->ev_begin : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
+      // a kernel that follows another group's kernel on its stream starts
+      // only once that kernel is done (no early set-up holding SMs)
+      t_pdl = pdl && (last_group[ls.slot] < 0 || last_group[ls.slot] == ls.group);
+      last_group[ls.slot] = ls.group;
       t_prio = ls.prio;
       if (ls.n == 1) {
         const int i = ls.members[0];
@@ -823,18 +858,14 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
         st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream, ls.scale);
       }
       t_prio = kNoPriority;
+      t_pdl = pdl;
       if (st != GOLDY_OK) return st;
       st = hook(opts ? opts->ev_end : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
     }
-    if (side) {
-      for (int k = 1; k < GOLDY_MAX_STREAMS; ++k)
-        if (side >> k & 1) {
-          cudaError_t e = enq_event_record(rt->join[k], static_cast<cudaStream_t>(streams[k]));
-          if (e == cudaSuccess) e = enq_wait(main, rt->join[k]);
-          if (e != cudaSuccess) return cuda_fail(e, "join event");
-        }
-    }
+    st = join(side);
+    if (st != GOLDY_OK) return st;
+    t0 = t1;
   }
   t_trace = nullptr;
   t_trace_ctas = 0;
