@@ -37,11 +37,13 @@ struct Runtime {
   void* green = nullptr;   // green context the events were created under (null: the device's own)
   cudaEvent_t fork = nullptr;
   cudaEvent_t join[GOLDY_MAX_STREAMS] = {};
+  cudaEvent_t started = nullptr;   // launch completion of a fused run's lead launch
 };
 
 void runtime_release(Runtime* rt) {
   if (!rt) return;
   if (rt->fork) cudaEventDestroy(rt->fork);
+  if (rt->started) cudaEventDestroy(rt->started);
   for (cudaEvent_t e : rt->join)
     if (e) cudaEventDestroy(e);
   delete rt;
@@ -63,6 +65,7 @@ struct Op {
   int cluster = 0;
   bool pdl = false;                  // programmatic dependency on the previous kernel of the stream
   int prio = kNoPriority;            // launch priority (kNoPriority: the stream's)
+  cudaEvent_t started = nullptr;     // launch-completion event to trigger (null: none)
   std::vector<uint64_t> params;      // 8-byte-aligned copy of the parameter block
   void* ptr = nullptr;
   size_t pitch = 0, width = 0, height = 0;
@@ -79,6 +82,9 @@ thread_local bool t_pdl = true;
 // A heterogeneous fused wave ranks its launches by work so the block
 // scheduler hands SMs to the largest first and the others fill its tail.
 thread_local int t_prio = kNoPriority;
+// Event the next GO-Kernel launch triggers once all of its CTAs have begun
+// (null: none); see the lead launch of a fused run in run_impl.
+thread_local cudaEvent_t t_started = nullptr;
 }
 
 namespace {
@@ -175,17 +181,24 @@ goldy_status kernel_setup(DeviceState& d, int kind, int out_bf16, int fused, int
 // Launch `fn` with one parameter block; as clusters of `cluster` CTAs when
 // cluster > 1.
 cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, void* params,
-                              int cluster, unsigned block = kThreads, bool pdl = false, int prio = kNoPriority) {
+                              int cluster, unsigned block = kThreads, bool pdl = false, int prio = kNoPriority,
+                              cudaEvent_t started = nullptr) {
   void* args[] = {params};
-  if (cluster <= 1 && !pdl && prio == kNoPriority)
+  if (cluster <= 1 && !pdl && prio == kNoPriority && !started)
     return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, stream);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(block);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[3];
+  cudaLaunchAttribute attr[4];
   unsigned n = 0;
+  if (started) {
+    attr[n].id = cudaLaunchAttributeLaunchCompletionEvent;
+    attr[n].val.launchCompletionEvent.event = started;
+    attr[n].val.launchCompletionEvent.flags = 0;
+    ++n;
+  }
   if (prio != kNoPriority) {
     attr[n].id = cudaLaunchAttributePriority;
     attr[n].val.priority = prio;
@@ -212,7 +225,8 @@ cudaError_t launch_kernel_now(const void* fn, unsigned grid, size_t smem, cudaSt
 cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream_t stream, const void* params,
                           size_t params_size, int cluster) {
   if (!t_rec)
-    return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster, kThreads, t_pdl, t_prio);
+    return launch_kernel_now(fn, grid, smem, stream, const_cast<void*>(params), cluster, kThreads, t_pdl, t_prio,
+                             t_started);
   Op op;
   op.kind = Op::kKernel;
   op.stream = stream;
@@ -222,6 +236,7 @@ cudaError_t launch_kernel(const void* fn, unsigned grid, size_t smem, cudaStream
   op.cluster = cluster;
   op.pdl = t_pdl;
   op.prio = t_prio;
+  op.started = t_started;
   op.params.resize((params_size + 7) / 8);
   std::memcpy(op.params.data(), params, params_size);
   t_rec->push_back(std::move(op));
@@ -288,7 +303,7 @@ cudaError_t replay(const Op& op) {
   switch (op.kind) {
     case Op::kKernel:
       return launch_kernel_now(op.fn, op.grid, op.smem, op.stream, const_cast<uint64_t*>(op.params.data()),
-                               op.cluster, op.block ? op.block : kThreads, op.pdl, op.prio);
+                               op.cluster, op.block ? op.block : kThreads, op.pdl, op.prio, op.started);
     case Op::kMemset2D: return cudaMemset2DAsync(op.ptr, op.pitch, 0, op.width, op.height, op.stream);
     case Op::kEventRecord: return cudaEventRecord(op.ev, op.stream);
     case Op::kEventRecordExternal: return cudaEventRecordWithFlags(op.ev, op.stream, 0);
@@ -647,6 +662,7 @@ Runtime* new_runtime(int dev, void* green, goldy_status* st) {
   rt->device = dev;
   rt->green = green;
   cudaError_t e = cudaEventCreateWithFlags(&rt->fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&rt->started, cudaEventDisableTiming);
   for (int k = 0; k < GOLDY_MAX_STREAMS && e == cudaSuccess; ++k)
     e = cudaEventCreateWithFlags(&rt->join[k], cudaEventDisableTiming);
   if (e != cudaSuccess) {
@@ -829,21 +845,60 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
       }
     return GOLDY_OK;
   };
+  // Fused mode: when the first wave has several launches, its largest (the
+  // lead) goes out first and triggers rt->started once all of its CTAs have
+  // begun; every other stream waits for that before its first launch.
+  // Priorities alone do not order the start: CTAs of a single-CTA kernel take
+  // SMs one at a time as the previous run's CTAs leave, while a cluster of
+  // the pair kernel needs two neighbouring SMs free at once, so a smaller
+  // launch used to occupy the GPU first.  (The event is best effort: the
+  // others may start later, never before the lead has begun.  Inside a stream
+  // capture the graph edge it becomes waited for the whole lead kernel —
+  // hetero_pair replayed 54 -> 63 us — so captured runs go without it.)
+  size_t lead = sets.size();
+  cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+  if (fused && !t_rec) {
+    cudaError_t e = cudaStreamIsCapturing(main, &capturing);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamIsCapturing");
+  }
+  if (fused && capturing == cudaStreamCaptureStatusNone) {
+    int kernels = 0;
+    for (size_t t = 0; t < sets.size() && sets[t].group == 0 && sets[t].wave == 0; ++t)
+      if (!sets[t].degenerate) {
+        ++kernels;
+        if (sets[t].rank == 0) lead = t;
+      }
+    if (kernels < 2) lead = sets.size();
+  }
+  std::vector<size_t> order;
+  order.reserve(sets.size());
+  if (lead < sets.size()) order.push_back(lead);
+  for (size_t t = 0; t < sets.size(); ++t)
+    if (t != lead) order.push_back(t);
   const bool pdl = t_pdl;
   int last_group[GOLDY_MAX_STREAMS];
-  for (int k = 0; k < GOLDY_MAX_STREAMS; ++k) last_group[k] = -1;
-  for (size_t t0 = 0; t0 < sets.size();) {
+  bool waited[GOLDY_MAX_STREAMS];
+  for (int k = 0; k < GOLDY_MAX_STREAMS; ++k) {
+    last_group[k] = -1;
+    waited[k] = false;
+  }
+  for (size_t t0 = 0; t0 < order.size();) {
     // the launches dispatched between one fork and its join
     size_t t1 = t0;
-    while (t1 < sets.size() && (fused || sets[t1].group == sets[t0].group)) ++t1;
+    while (t1 < order.size() && (fused || sets[order[t1]].group == sets[order[t0]].group)) ++t1;
     uint32_t used = 0;
-    for (size_t t = t0; t < t1; ++t) used |= 1u << sets[t].slot;
+    for (size_t t = t0; t < t1; ++t) used |= 1u << sets[order[t]].slot;
     const uint32_t side = used & ~1u;            // slots other than 0 fork from and join into streams[0]
     st = fork(side);
     if (st != GOLDY_OK) return st;
     for (size_t t = t0; t < t1; ++t) {
-      const LaunchSet& ls = sets[t];
+      const LaunchSet& ls = sets[order[t]];
       cudaStream_t stream = static_cast<cudaStream_t>(streams[ls.slot]);
+      if (lead < sets.size() && order[t] != lead && !waited[ls.slot] && ls.slot != sets[lead].slot) {
+        cudaError_t e = enq_wait(stream, rt->started);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent (lead started)");
+        waited[ls.slot] = true;
+      }
       st = hook(opts ? opts->ev_begin : nullptr, ls.members, ls.n, stream);
       if (st != GOLDY_OK) return st;
       // a kernel that follows another group's kernel on its stream starts
@@ -851,6 +906,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
       t_pdl = pdl && (last_group[ls.slot] < 0 || last_group[ls.slot] == ls.group);
       last_group[ls.slot] = ls.group;
       t_prio = ls.prio;
+      t_started = order[t] == lead ? rt->started : nullptr;
       if (ls.n == 1) {
         const int i = ls.members[0];
         st = launch_gemm(*d, s->gemms[i], A[i], B[i], C[i], ws, stream, ls.scale);
@@ -858,6 +914,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
         st = launch_fused(*d, s, ls.members, ls.n, A, B, C, ws, stream, ls.scale);
       }
       t_prio = kNoPriority;
+      t_started = nullptr;
       t_pdl = pdl;
       if (st != GOLDY_OK) return st;
       st = hook(opts ? opts->ev_end : nullptr, ls.members, ls.n, stream);
