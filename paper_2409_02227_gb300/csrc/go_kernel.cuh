@@ -143,6 +143,34 @@ __device__ __forceinline__ UnitCoord decode_unit(const LaunchParams<MAXG>& p, in
   return c;
 }
 
+// The fields of a GemmWork that decode a unit, copied into shared memory at
+// set-up: the kernel parameter block is several kilobytes (tensor maps
+// first), and reading these fields from it on the producer's critical path
+// measured ~0.4 us before the first load of a launch.
+struct UnitTable {
+  int32_t unit_begin, split, tiles_m, tiles_n, k_blocks;
+};
+
+__device__ __forceinline__ UnitCoord decode_unit_tab(const UnitTable* t, int n_gemms, int u) {
+  UnitCoord c;
+  int g = 0;
+#pragma unroll 1
+  while (g + 1 < n_gemms && u >= t[g + 1].unit_begin) ++g;
+  const UnitTable& w = t[g];
+  const int local = u - w.unit_begin;
+  c.g = g;
+  c.tile = local / w.split;
+  c.s = local - c.tile * w.split;
+  const int per_batch = w.tiles_m * w.tiles_n;
+  c.b = c.tile / per_batch;
+  const int t2 = c.tile - c.b * per_batch;
+  c.tm = t2 % w.tiles_m;
+  c.tn = t2 / w.tiles_m;
+  c.kb0 = (c.s * w.k_blocks) / w.split;
+  c.kb1 = ((c.s + 1) * w.k_blocks) / w.split;
+  return c;
+}
+
 __device__ __forceinline__ void trace_stamp(unsigned long long* trace, int slot) {
   if (trace) trace[blockIdx.x * kTracePerCta + slot] = ptx::global_timer();
 }
@@ -506,6 +534,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
+  UnitTable* utab = reinterpret_cast<UnitTable*>(tmem_slot + 4);   // MAXG entries, inside the 1 KB barrier area
+  static_assert((2 * STAGES + 2 * ACC + 4) * 8 + 16 + MAXG * int(sizeof(UnitTable)) <= 1024, "barrier area");
+  const int n_gemms = p.n_gemms;
 
   const uint32_t tiles_base = ptx::smem_u32(smem);
   const int warp = threadIdx.x >> 5;
@@ -560,6 +591,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   if (warp == 1) {
     ptx::tmem_alloc(ptx::smem_u32(tmem_slot), TMEM_COLS);
     ptx::tmem_relinquish();
+  } else if (warp == 2) {
+    for (int g = lane; g < p.n_gemms; g += 32) {
+      UnitTable e;
+      e.unit_begin = p.g[g].unit_begin;
+      e.split = p.g[g].split;
+      e.tiles_m = p.g[g].tiles_m;
+      e.tiles_n = p.g[g].tiles_n;
+      e.k_blocks = p.g[g].k_blocks;
+      utab[g] = e;
+    }
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -582,13 +623,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       bool ok = true;
       for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
         if (issued == 0) trace_stamp(trace, kTrProducerGo);
-        const UnitCoord c = decode_unit(p, u);
+        const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         const void* ta = &p.tmap_a[c.g];
         const void* tb = &p.tmap_b[c.g];
         const int m0 = c.tm * TILE_M;
         const int n0 = c.tn * TILE_N;
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
-          if (!ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+          // a slot is waited for only once it has been filled before: on the
+          // first pass the ring is empty (waiting on a fresh barrier's
+          // preceding phase measured ~0.7 us before the first load)
+          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
             ok = false;
             break;
           }
@@ -626,14 +670,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     if (lane == 0) {
       // ---------------------------------------------------------- MMA issuer
       int stage = 0, acc = 0;
-      uint32_t phase = 0, acc_phase = 0;
+      uint32_t phase = 0, acc_phase = 0, acc_used = 0;
       bool ok = true, any = false;
       for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
-        const UnitCoord c = decode_unit(p, u);
-        if (!ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+        const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
+        // an accumulator is waited for only once it has been used before
+        if ((acc_used >> acc & 1) && !ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
           ok = false;
           break;
         }
+        acc_used |= 1u << acc;
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + uint32_t(acc * MMA_N);
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
@@ -691,7 +737,11 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     uint32_t stg = 0;                       // staging buffers used (TMA-store epilogue)
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
     for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
-      const UnitCoord c = decode_unit(p, u);
+      const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
+      // the GEMM's output description, read from the parameter block while
+      // the accumulator is still being computed
+      const GemmWork w = p.g[c.g];
+      const CView cv = c_view<OUT_BF16>(w, c.b);
       bool released = false;                // accumulator already handed back
       bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
       ok = ptx::named_bar_and(1, 128, ok);
@@ -702,8 +752,6 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       ptx::tc_fence_after();
       const bool first_unit = (u == int(blockIdx.x));
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
-      const GemmWork& w = p.g[c.g];
-      const CView cv = c_view<OUT_BF16>(w, c.b);
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);

@@ -113,7 +113,8 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         const int m0 = c.tm * 256 + int(rank) * 128;
         const int n0 = c.tn * 256 + int(rank) * HALF_N;
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
-          if (!ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+          // only a slot filled before is waited for (see go_gemm_kernel)
+          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
             ok = false;
             break;
           }
@@ -156,16 +157,19 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     if (lane == 0 && lead) {
       // ------------------------------------------------- MMA issuer (even CTA)
       int stage = 0, acc = 0;
-      uint32_t phase = 0, acc_phase = 0;
+      uint32_t phase = 0, acc_phase = 0, acc_used = 0;
       bool ok = true, any = false;
       for (int u = pair; ok && u < p.total_units; u += n_pairs) {
         const UnitCoord c = decode_unit(p, u);
         // both CTAs drained this accumulator (the odd CTA signals with a
-        // cluster-scope release, so wait with a cluster-scope acquire)
-        if (!ptx::mbar_wait_cluster(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+        // cluster-scope release, so wait with a cluster-scope acquire); the
+        // first use of an accumulator needs no wait
+        if ((acc_used >> acc & 1) &&
+            !ptx::mbar_wait_cluster(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
           ok = false;
           break;
         }
+        acc_used |= 1u << acc;
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + uint32_t(acc * 256);
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
