@@ -49,6 +49,9 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  UnitTable* utab = reinterpret_cast<UnitTable*>(tmem_slot + 4);   // see go_gemm_kernel
+  static_assert((2 * STAGES + 2 * ACC + 1) * 8 + 16 + MAXG * int(sizeof(UnitTable)) <= 1024, "barrier area");
+  const int n_gemms = p.n_gemms;
 
   const uint32_t tiles_base = ptx::smem_u32(smem);
   const int warp = threadIdx.x >> 5;
@@ -90,6 +93,16 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   if (warp == 1) {
     ptx::tmem_alloc_pair(ptx::smem_u32(tmem_slot), TMEM_COLS);
     ptx::tmem_relinquish_pair();
+  } else if (warp == 2) {
+    for (int g = lane; g < p.n_gemms; g += 32) {
+      UnitTable e;
+      e.unit_begin = p.g[g].unit_begin;
+      e.split = p.g[g].split;
+      e.tiles_m = p.g[g].tiles_m;
+      e.tiles_n = p.g[g].tiles_n;
+      e.k_blocks = p.g[g].k_blocks;
+      utab[g] = e;
+    }
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -107,7 +120,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       uint32_t phase = 0, issued = 0, last_phase = 0;
       bool ok = true;
       for (int u = pair; ok && u < p.total_units; u += n_pairs) {
-        const UnitCoord c = decode_unit(p, u);
+        const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         const void* ta = &p.tmap_a[c.g];
         const void* tb = &p.tmap_b[c.g];
         const int m0 = c.tm * 256 + int(rank) * 128;
@@ -160,7 +173,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       uint32_t phase = 0, acc_phase = 0, acc_used = 0;
       bool ok = true, any = false;
       for (int u = pair; ok && u < p.total_units; u += n_pairs) {
-        const UnitCoord c = decode_unit(p, u);
+        const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         // both CTAs drained this accumulator (the odd CTA signals with a
         // cluster-scope release, so wait with a cluster-scope acquire); the
         // first use of an accumulator needs no wait
@@ -220,7 +233,9 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     uint32_t stg = 0;
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
     for (int u = pair; u < p.total_units; u += n_pairs) {
-      const UnitCoord c = decode_unit(p, u);
+      const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
+      const GemmWork w = p.g[c.g];                 // read while the accumulator is computed
+      const CView cv = c_view<OUT_BF16>(w, c.b);
       bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
       ok = ptx::named_bar_and(1, 128, ok);
       if (!ok) {
@@ -230,8 +245,6 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       ptx::tc_fence_after();
       const bool first_unit = (u == pair);
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
-      const GemmWork& w = p.g[c.g];
-      const CView cv = c_view<OUT_BF16>(w, c.b);
       const int m0 = c.tm * 256 + int(rank) * 128;
       const int n0 = c.tn * 256;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
