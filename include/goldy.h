@@ -97,8 +97,15 @@ typedef struct goldy_graph goldy_graph;
  * group, the GEMMs that run at the same time (a "wave" of CD members) and
  * share a kernel kind and output dtype go into ONE persistent launch over the
  * concatenation of their tiles (at most 16 GEMMs per launch); its grid cap is
- * the sum of the members' caps.  Without it every GEMM is its own launch on
- * its slot's stream.  The plan (groups, CDs, variants, slots) is the same. */
+ * the sum of the members' caps.  A wave's launches carry launch priorities
+ * ranked by their FLOPs, and the first wave's largest launch goes out first
+ * (outside a stream capture the other streams also wait until all of its
+ * CTAs have begun).  Groups are not separated by a join: the run forks once
+ * and joins once, and a later group's launches take lower priorities, so they
+ * fill the SMs an earlier group frees.  Without FUSED every GEMM is its own
+ * launch on its slot's stream and the groups run one after another.  The plan
+ * (groups, CDs, variants, slots) is the same, and so are the results, byte
+ * for byte. */
 #define GOLDY_PLAN_FUSED 0x10
 
 #define GOLDY_MAX_GEMMS 64      /* GEMMs per plan */

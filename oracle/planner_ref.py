@@ -242,14 +242,15 @@ def preferred_cd(speedup: dict, gain: float = 0.05, near: float = 0.01) -> int:
     """Preferred CD from measured speedups over serial execution (Sec. 4.3:
     the CD with the most speedup; Sec. 5.4: sequential unless some CD gains at
     least 5%).  Among CDs whose speedup is within ``near`` (relative) of the
-    best, the smallest wins.  ``speedup[1]`` is 1 by definition."""
+    best, the largest wins (the paper does not address near-ties).
+    ``speedup[1]`` is 1 by definition."""
     cands = {cd: s for cd, s in speedup.items() if cd in CD_CLASSES and cd != 1}
     if not cands:
         return 1
     best = max(cands.values())
     if best < 1.0 + gain:
         return 1
-    return min(cd for cd, s in cands.items() if s >= best * (1.0 - near))
+    return max(cd for cd, s in cands.items() if s >= best * (1.0 - near))
 
 
 def corun_plan(d: Desc, lut_bytes: bytes, policy: int) -> Tuple[int, int, int]:

@@ -804,6 +804,50 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
         if (!sets[t1].degenerate) ++kernels;
         ++t1;
       }
+      // A plan of one group: the wave is bounded by the largest uniform scale
+      // (at most c/m) at which its launches are all resident at once, since
+      // over-subscribing left the lower-priority launch of a small wave
+      // waiting for SMs (a two-GEMM set: 14.4 -> 10.5 us with the bound).
+      // Plans of several groups keep the full c/m: there the same bound
+      // measured 5-28% slower (the over-subscribed first group's CTAs take
+      // SMs as they free up, ahead of the later groups' launches).
+      double fit = 1e30;
+      if (kernels > 1 && !soft_groups) {
+        struct Need {
+          double units, cap, ctas;   // CTAs of work, the launch's own cap, CTAs per SM
+        };
+        std::vector<Need> need;
+        for (size_t t = t0; t < t1; ++t) {
+          if (sets[t].degenerate) continue;
+          const GemmPlan& g0 = s->gemms[sets[t].members[0]];
+          int ctas = 0;
+          st = kernel_setup(*d, g0.kind, g0.desc.c_dtype == GOLDY_BF16 ? 1 : 0, sets[t].n > 1 ? 1 : 0, &ctas);
+          if (st != GOLDY_OK) return st;
+          Need nd{0.0, 0.0, double(ctas)};
+          for (int j = 0; j < sets[t].n; ++j) {
+            const GemmPlan& gp = s->gemms[sets[t].members[j]];
+            nd.units += double(gp.units) * (kKinds[gp.kind].pair ? 2.0 : 1.0);
+            nd.cap += std::max(1.0, double(ctas) * sms(*d) / variant_of(gp.variant).rc_div);
+          }
+          need.push_back(nd);
+        }
+        auto sm_use = [&](double sc) {
+          double u = 0.0;
+          for (const Need& nd : need) u += std::min(nd.units, std::min(nd.cap * sc, nd.ctas * sms(*d))) / nd.ctas;
+          return u;
+        };
+        if (sm_use(1.0) <= double(sms(*d))) {
+          double lo = 1.0, hi = double(wave_size);
+          if (sm_use(hi) <= double(sms(*d))) lo = hi;
+          for (int it = 0; it < 30 && hi - lo > 1e-3; ++it) {
+            const double mid = 0.5 * (lo + hi);
+            (sm_use(mid) <= double(sms(*d)) ? lo : hi) = mid;
+          }
+          fit = lo;
+        } else {
+          fit = 1.0;
+        }
+      }
       for (size_t t = t0; t < t1; ++t) {
         if (sets[t].degenerate) continue;
         for (size_t u = t0; u < t1; ++u)
@@ -811,7 +855,7 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
               (sets[u].flops > sets[t].flops || (sets[u].flops == sets[t].flops && u < t)))
             ++sets[t].rank;
         if (kernels > 1) {
-          sets[t].scale = double(wave_size) / double(sets[t].n);
+          sets[t].scale = std::min(double(wave_size) / double(sets[t].n), std::max(1.0, fit));
           sets[t].prio = level(sets[t].rank);
         }
         // groups of a fused plan are not separated by a join: group g's
@@ -868,7 +912,10 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
         ++kernels;
         if (sets[t].rank == 0) lead = t;
       }
-    if (kernels < 2) lead = sets.size();
+    // only a pair-kernel lead needs it (its clusters need two free SMs at
+    // once); for single-CTA launches the priorities suffice, and the event
+    // and waits measured ~4 us on a two-GEMM set of small kernels
+    if (kernels < 2 || (lead < sets.size() && !kKinds[s->gemms[sets[lead].members[0]].kind].pair)) lead = sets.size();
   }
   std::vector<size_t> order;
   order.reserve(sets.size());

@@ -21,8 +21,13 @@ list:
          CD gains at least 5% (Sec. 5.4); CDs within 1% of the best go to the
          smaller one.
 
-Each bucket (floor log2 of M, N, K; output dtype) is profiled at its lower
-edge (M, N, K = powers of two), where DNN layer sizes usually sit.  Timing:
+Each bucket (floor log2 of M, N, K; output dtype) is profiled at two
+points: its lower edge (M, N, K = powers of two), where DNN layer sizes
+usually sit, and its geometric centre (2^(l + 1/2), N and K rounded to 64).
+A candidate's score is its mean time relative to the fastest candidate at
+each point, and speedups are averaged over the points, so that a choice holds
+across the bucket (a table profiled at the lower edges alone ran the
+randomized sets, whose shapes fill the buckets, 7% slower).  Timing:
 prepared runs (recorded plain launches, the way the benchmark replays a step)
 back to back on one stream, as the paper ran GEMMs back to back on each
 stream (Sec. 5.3), rotating over disjoint copies of the operands so that they
@@ -78,22 +83,46 @@ def write_lut(entries, n_variants: int, sm_count: int) -> bytes:
 
 def preferred_cd(speedup: Dict[int, float], gain: float = 0.05, near: float = 0.01) -> int:
     """Largest-speedup CD, sequential unless the gain reaches ``gain``; CDs
-    within ``near`` of the best resolve to the smallest."""
+    within ``near`` of the best resolve to the largest (a larger CD costs no
+    more per GEMM on a near-tie, and lets a heterogeneous set run in fewer
+    groups: the planner merges keys only while each prefers the group's size)."""
     best_cd, best = 1, 1.0
     for cd in (2, 4, 8, 16):
         if cd in speedup and speedup[cd] > best:
             best_cd, best = cd, speedup[cd]
     if best < 1.0 + gain:
         return 1
-    for cd in (2, 4, 8, 16):
+    for cd in (16, 8, 4, 2):
         if cd in speedup and speedup[cd] >= best * (1.0 - near):
             return cd
     return best_cd
 
 
+def logged_pref(rec: dict) -> int:
+    """Preferred CD of a logged bucket under the current rule."""
+    return preferred_cd({int(c): v for c, v in rec["speedup"].items()})
+
+
 def bucket_shape(key) -> Tuple[int, int, int, int]:
     lm, ln, lk, out = key
     return 1 << lm, max(64, 1 << ln), max(64, 1 << lk), out
+
+
+def bucket_centre(key) -> Tuple[int, int, int, int]:
+    """Geometric centre of a bucket: 2^(l + 1/2) per size, N and K rounded to
+    multiples of 64 (as the workloads' N and K are)."""
+    lm, ln, lk, out = key
+    c = lambda l: 2.0 ** (l + 0.5)
+    return (max(1, int(round(c(lm)))), max(64, 64 * int(round(c(ln) / 64))), max(64, 64 * int(round(c(lk) / 64))),
+            out)
+
+
+def bucket_points(key) -> List[Tuple[int, int, int, int]]:
+    """Sample points a bucket is profiled at: its lower edge and its centre."""
+    pts = [bucket_shape(key)]
+    if bucket_centre(key) != pts[0]:
+        pts.append(bucket_centre(key))
+    return pts
 
 
 def candidates(M: int, N: int, K: int, sm_count: int) -> List[Tuple[int, int]]:
@@ -183,40 +212,43 @@ class Bench:
 
 
 def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) -> dict:
-    M, N, K, out = bucket_shape(key)
-    bench = Bench(M, N, K, out, partition=partition)
-    cands = candidates(M, N, K, sm_count)
+    """Steps 1 and 2 for one bucket, at each of its sample points; a variant's
+    score is its mean time relative to the fastest candidate at each point,
+    so that the choice holds across the bucket, not at one shape only."""
+    points = bucket_points(key)
+    M, N, K, out = points[0]
+    benches = [Bench(*pt, partition=partition) for pt in points]
+    cands = sorted(set().union(*[set(candidates(pt[0], pt[1], pt[2], sm_count)) for pt in points]))
     rows = []
+
+    def best_of(variants, copies, step, extra):
+        times = {v: [b.time_us(v, copies, True, fused=fused) for b in benches] for v in variants}
+        for v, ts in times.items():
+            for pi, t in enumerate(ts):
+                rows.append(dict(step=step, variant=v, point=pi, us=t, **extra))
+        fastest = [min(ts[pi] for ts in times.values()) for pi in range(len(points))]
+        score = {v: sum(t / f for t, f in zip(ts, fastest)) / len(points) for v, ts in times.items()}
+        v = min(variants, key=lambda x: (score[x], x))
+        return v, times[v]
+
     winners = {}
     for rc in RC_DIVS:                                  # step 1
-        best = None
-        for kind, split in cands:
-            v = G.variant_id(kind, split, rc)
-            t = bench.time_us(v, 1, True, fused=fused)
-            rows.append({"step": 1, "rc": rc, "variant": v, "us": t})
-            if best is None or t < best[0]:
-                best = (t, v)
-        winners[rc] = best
-    go = {1: winners[1][1]}
-    t_cd = {1: winners[1][0]}
+        winners[rc] = best_of([G.variant_id(kind, split, rc) for kind, split in cands], 1, 1, {"rc": rc})
+    go = {1: winners[1][0]}
+    t_cd = {1: winners[1][1]}
     for cd in (2, 4, 8, 16):                            # step 2
-        best = None
-        for rc in RC_DIVS:
-            v = winners[rc][1]
-            t = bench.time_us(v, cd, True, fused=fused)
-            rows.append({"step": 2, "cd": cd, "rc": rc, "variant": v, "us": t})
-            if best is None or t < best[0]:
-                best = (t, v)
-        go[cd] = best[1]
-        t_cd[cd] = best[0]
-    speedup = {cd: cd * t_cd[1] / t_cd[cd] for cd in CD_CLASSES}
+        go[cd], t_cd[cd] = best_of(sorted({winners[rc][0] for rc in RC_DIVS}), cd, 2, {"cd": cd})
+    # speedup over running the copies one after another, averaged over the points
+    speedup = {cd: sum(cd * t1 / tc for t1, tc in zip(t_cd[1], t_cd[cd])) / len(points) for cd in CD_CLASSES}
     pref = preferred_cd(speedup)
-    rec = {"key": list(key), "shape": [M, N, K, out], "pref_cd": pref, "launch": "fused" if fused else "streams",
-           "variants": [go[c] for c in CD_CLASSES], "t_us": {str(c): t_cd[c] for c in CD_CLASSES},
+    rec = {"key": list(key), "shape": [M, N, K, out], "points": [list(pt) for pt in points], "pref_cd": pref,
+           "launch": "fused" if fused else "streams", "variants": [go[c] for c in CD_CLASSES],
+           "t_us": {str(c): t_cd[c][0] for c in CD_CLASSES},
+           "t_us_points": {str(c): t_cd[c] for c in CD_CLASSES},
            "speedup": {str(c): speedup[c] for c in CD_CLASSES}, "rows": rows}
     log.write(json.dumps(rec) + "\n")
     log.flush()
-    del bench
+    del benches
     torch.cuda.empty_cache()
     return rec
 
@@ -308,8 +340,9 @@ def add_corun_flags(out_dir: str, fused: bool, partition=None) -> None:
             if i % 20 == 0:
                 print(f"[corun {i + 1}/{len(recs)}] {key} {t}", flush=True)
     sm_count = struct.unpack_from("<I", open(os.path.join(out_dir, "goldy_lut.bin"), "rb").read(), 20)[0]
-    # flags re-derived from the logged times, so a resumed log follows the current rule
-    entries = [(k, r["pref_cd"], r["variants"], corun_flags(done[k]["t_us"])) for k, r in recs.items()]
+    # preferences and flags re-derived from the logged speedups and times, so
+    # the table follows the current rules
+    entries = [(k, logged_pref(r), r["variants"], corun_flags(done[k]["t_us"])) for k, r in recs.items()]
     lut = write_lut(entries, G.goldy_variant_count(), sm_count)
     G.goldy_lut_from_memory(lut)
     with open(os.path.join(out_dir, "goldy_lut.bin"), "wb") as f:
@@ -442,7 +475,7 @@ def main(argv=None) -> int:
             done[key] = rec
             print(f"[{i + 1}/{len(keys)}] {key} shape {rec['shape']} pref {rec['pref_cd']} "
                   f"variants {rec['variants']} ({time.time() - tb:.1f}s)", flush=True)
-    entries = [(k, r["pref_cd"], r["variants"]) for k, r in done.items()]
+    entries = [(k, logged_pref(r), r["variants"]) for k, r in done.items()]
     lut = write_lut(entries, G.goldy_variant_count(), sm_count)
     G.goldy_lut_from_memory(lut)          # validate with the library's own parser
     with open(os.path.join(args.out, "goldy_lut.bin"), "wb") as f:

@@ -376,3 +376,56 @@ def test_dependent_launches_see_the_previous_kernels_output(cuda_ok, fused):
         check_close(outs[False][j], prev, bs[j], f"chain step {j}")
         prev = outs[False][j]
         assert torch.equal(outs[False][j].view(torch.int16), outs[True][j].view(torch.int16))
+
+
+def _multi_group_sweep_sets(lut, count):
+    """The first `count` randomized sets whose plan has several groups."""
+    found = []
+    for j in range(wl.SWEEP_SETS):
+        _, specs, _ = wl.sweep_specs(j)
+        descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in specs]
+        if G.goldy_schedule_query(G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED))[1] > 1:
+            found.append(j)
+            if len(found) == count:
+                break
+    return found
+
+
+@pytest.mark.parametrize("pick", [0, 1])
+def test_fused_dispatch_matches_strict_groups(cuda_ok, pick):
+    # A multi-group plan in fused mode (one fork and join, groups ordered by
+    # launch priority, the first wave's largest launch first) against the
+    # same plan in streams mode (groups one after another): same bytes, run
+    # eagerly, as a prepared run and as a CUDA graph.
+    lut = G.goldy_lut_load(G.DEFAULT_LUT)
+    picks = _multi_group_sweep_sets(lut, 2)
+    assert len(picks) == 2, "want randomized sets whose plan has several groups"
+    j = picks[pick]
+    st = wl.make_sweep_set(j)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    fused = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    strict = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO)
+    outs = [s.out_dtype for s in st.specs]
+    Ls = Launch(strict, st.a, st.b, outs)
+    Ls.run()
+    ref = Ls.results()
+    Lf = Launch(fused, st.a, st.b, outs)
+    Lf.run()
+    runs = [Lf.results()]
+    for make in (Lf.exec, Lf.graph):
+        for c in Lf.dC:
+            c.fill_(float("nan"))
+        handle = make()
+        if make == Lf.exec:
+            G.goldy_exec_launch(handle)
+        else:
+            G.goldy_graph_launch(handle, Lf.streams[0].cuda_stream)
+        torch.cuda.current_stream().wait_stream(Lf.streams[0])
+        runs.append(Lf.results())
+        del handle
+    for got in runs:
+        for i in range(len(descs)):
+            x, y = got[i], ref[i]
+            if x.dtype == torch.bfloat16:
+                x, y = x.view(torch.int16), y.view(torch.int16)
+            assert torch.equal(x, y), f"sweep {j} gemm {i}"

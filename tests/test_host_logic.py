@@ -40,6 +40,13 @@ def test_lut_writer_matches_oracle_format():
 
 def test_bucket_shapes_and_candidates():
     assert P.bucket_shape((7, 10, 12, 0)) == (128, 1024, 4096, 0)
+    # centre 2^(l + 1/2): 128 * sqrt2 = 181.02, 1024 * sqrt2 = 1448.2 -> 64 * 23, 4096 * sqrt2 = 5792.6 -> 64 * 91
+    assert P.bucket_centre((7, 10, 12, 0)) == (181, 1472, 5824, 0)
+    assert P.bucket_points((7, 10, 12, 0)) == [(128, 1024, 4096, 0), (181, 1472, 5824, 0)]
+    # every centre lies inside its bucket
+    for key in [(4, 8, 9, 1), (11, 13, 11, 0), (6, 12, 8, 1)]:
+        M, N, K, _ = P.bucket_centre(key)
+        assert (M.bit_length() - 1, N.bit_length() - 1, K.bit_length() - 1) == key[:3]
     c = P.candidates(32, 4096, 1024, 152)
     kinds = {k for k, _ in c}
     assert {6, 7, 8, 9} <= kinds                      # transposed tiles offered for skinny M

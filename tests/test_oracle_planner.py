@@ -159,7 +159,9 @@ def test_schedule_bytes_by_hand():
 def test_preferred_cd_rule():
     assert pr.preferred_cd({1: 1.0, 2: 1.04, 4: 1.049}) == 1         # below 5%
     assert pr.preferred_cd({1: 1.0, 2: 1.05}) == 2
-    assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.105}) == 2         # within 1% -> smaller
+    assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.105}) == 4         # the best
+    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.195}) == 4         # within 1% of the best -> larger
+    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.18, 8: 1.195}) == 8   # 4 is 1.7% off, 8 within 1%
     assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.20, 8: 1.15}) == 4
     assert pr.preferred_cd({1: 1.0, 2: 0.8, 16: 1.9}) == 16
     assert pr.preferred_cd({1: 1.0}) == 1

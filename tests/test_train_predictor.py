@@ -59,9 +59,13 @@ def test_separable_data_fitted_perfectly():
 
 
 def test_label_rule():
-    # speedups 1, 1.9, 3.0, 3.02, 2.0 -> 4 and 8 within 1% -> 4
+    # speedups 1, 1.9, 3.0, 3.02, 2.0 -> 4 and 8 within 1% -> the larger, 8
     t = {1: 10.0, 2: 2 * 10 / 1.9, 4: 4 * 10 / 3.0, 8: 8 * 10 / 3.02, 16: 16 * 10 / 2.0}
-    assert T.label_of(t) == 4
+    assert T.label_of(t) == 8
+    # 3.0 vs 3.1: 4 is more than 1% off the best -> 8
+    assert T.label_of({1: 10.0, 2: 2 * 10 / 1.9, 4: 4 * 10 / 3.0, 8: 8 * 10 / 3.1, 16: 16 * 10 / 2.0}) == 8
+    # 3.1 vs 3.0: 8 is more than 1% off the best -> 4
+    assert T.label_of({1: 10.0, 2: 2 * 10 / 1.9, 4: 4 * 10 / 3.1, 8: 8 * 10 / 3.0, 16: 16 * 10 / 2.0}) == 4
     assert T.label_of(t, available=2) == 2
     # best gain below 5% -> sequential
     assert T.label_of({1: 10.0, 2: 2 * 10 / 1.04, 4: 40.0, 8: 80.0, 16: 160.0}) == 1
