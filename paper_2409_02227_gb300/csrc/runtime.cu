@@ -804,10 +804,11 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
         if (!sets[t1].degenerate) ++kernels;
         ++t1;
       }
-      // A plan of one group: the wave is bounded by the largest uniform scale
-      // (at most c/m) at which its launches are all resident at once, since
-      // over-subscribing left the lower-priority launch of a small wave
-      // waiting for SMs (a two-GEMM set: 14.4 -> 10.5 us with the bound).
+      // A plan of one group whose wave fits on the GPU unscaled: the scale is
+      // bounded by the largest uniform one (at most c/m) at which its launches
+      // are all resident at once, since over-subscribing left the
+      // lower-priority launch of a small wave waiting for SMs (a two-GEMM
+      // set: 14.4 -> 10.5 us with the bound).
       // Plans of several groups keep the full c/m: there the same bound
       // measured 5-28% slower (the over-subscribed first group's CTAs take
       // SMs as they free up, ahead of the later groups' launches).
@@ -836,6 +837,9 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
           for (const Need& nd : need) u += std::min(nd.units, std::min(nd.cap * sc, nd.ctas * sms(*d))) / nd.ctas;
           return u;
         };
+        // (a wave that over-subscribes the GPU unscaled keeps c/m: its smaller
+        // launches run in the largest one's tail, where a quarter-GPU cap
+        // left one at two rounds — 160 -> 194 us on a four-GEMM set)
         if (sm_use(1.0) <= double(sms(*d))) {
           double lo = 1.0, hi = double(wave_size);
           if (sm_use(hi) <= double(sms(*d))) lo = hi;
@@ -844,8 +848,6 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
             (sm_use(mid) <= double(sms(*d)) ? lo : hi) = mid;
           }
           fit = lo;
-        } else {
-          fit = 1.0;
         }
       }
       for (size_t t = t0; t < t1; ++t) {
