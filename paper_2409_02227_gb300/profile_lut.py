@@ -423,6 +423,8 @@ def main(argv=None) -> int:
                     help="tune inside an SM partition (green context) of at least SMS SMs (0: the whole GPU "
                          "as a partition); grid caps and the table's SM count follow the partition")
     ap.add_argument("--scaling-keys", action="store_true", help="buckets of the GPU-scaling study's sets")
+    ap.add_argument("--batched-keys", action="store_true",
+                    help="buckets of the batched study's B-GEMMs (M x batch rows)")
     ap.add_argument("--corun-flags", action="store_true",
                     help="step 3 over the table already profiled in --out: set each bucket's co-run flag")
     ap.add_argument("--configs", action="store_true", help="buckets of the fixed workload sets")
@@ -448,6 +450,9 @@ def main(argv=None) -> int:
         keys += sweep_keys()
     if args.scaling_keys:
         keys += sorted({bucket_of(*sh) for sh in wl.scaling_study_shapes()})
+    if args.batched_keys:
+        keys += sorted({bucket_of(s.M * s.batch, s.N, s.K, s.out_dtype)
+                        for members in (2, 4) for i in range(16) for s in wl.batched_study_specs(i, members)[1]})
     keys += [tuple(int(x) for x in k.split(",")) for k in args.keys]
     keys = sorted(set(keys))
     log_path = os.path.join(args.out, "profile.jsonl")
