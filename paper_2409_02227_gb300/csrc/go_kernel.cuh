@@ -438,13 +438,22 @@ __device__ __forceinline__ void reduce_slice_dsmem(const CView& w, uint32_t part
   }
 }
 
+// Layout of a slice (R rows x MMA_N fp32 columns) of the pushed reduction:
+// column-chunk major, so that each 32-column chunk of a slice is one
+// contiguous R x 128-byte block that can be sent as soon as it is staged;
+// within a chunk, granule j of row rr sits at j ^ (rr & 7) (a thread writing
+// its row and a warp reading consecutive granules both spread over the banks).
+__device__ __forceinline__ uint32_t push_offset(int rr, int f, int R) {
+  return uint32_t((f >> 3) * R * 128 + rr * 128 + (((f & 7) ^ (rr & 7)) << 4));
+}
+
 // Cluster split-K with pushed partials: CTA s of the S splits of a tile owns
 // rows s*128/S .. (s+1)*128/S - 1.  Every CTA sends the rows it does not own
 // to their owner (a bulk copy into the owner's receive slot, counted on the
 // owner's mbarrier) and keeps its own rows in its ring; the owner then sums,
 // from its own shared memory, the S partials of its rows in split order
 // 0, 1, ..., S-1 and stores them.  A slot holds 128/S rows in the layout of
-// part_offset; sender s goes to slot s (s < owner) or s - 1 (s > owner).
+// push_offset; sender s goes to slot s (s < owner) or s - 1 (s > owner).
 template <int MMA_N, int S, bool SWAP, bool OUT_BF16>
 __device__ __forceinline__ void reduce_slice_pushed(const CView& w, uint32_t own_slot, uint32_t recv_slots, int rank,
                                                     int m0, int n0, int t) {
@@ -460,7 +469,7 @@ __device__ __forceinline__ void reduce_slice_pushed(const CView& w, uint32_t own
 #pragma unroll 2
   for (int k = 0; k < PER_THREAD; ++k) {
     const int i = t + 128 * k;
-    const uint32_t off = part_offset<MMA_N>(i / G4, i % G4);
+    const uint32_t off = push_offset(i / G4, i % G4, R);
     float4 v[S];
 #pragma unroll
     for (int s2 = 0; s2 < S; ++s2) v[s2] = ptx::ld_shared_v4(src[s2] + off);
@@ -773,11 +782,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         // ---- cluster split-K, pushed: one unit per CTA.  Row r of the
         // accumulator belongs to the CTA of rank r / (128/S).  The partial
         // goes into the ring (free once the accumulator is complete) as S
-        // slices of 128/S rows; one bulk copy per peer sends it its slice,
-        // counted on the peer's receive barrier.  Then wait until every
-        // peer's copy of this CTA's slice has landed and reduce the S slices
-        // from local shared memory.  The cluster barrier at kernel exit keeps
-        // every source buffer alive until its copies have landed.
+        // slices of 128/S rows, 32 columns at a time; as soon as a chunk is
+        // staged, one bulk copy per peer sends it that chunk of its slice,
+        // counted on the peer's receive barrier, while the next chunk is read
+        // out of tensor memory.  Then wait until every peer's copies of this
+        // CTA's slice have landed and reduce the S slices from local shared
+        // memory.  The cluster barrier at kernel exit keeps every source
+        // buffer alive until its copies have landed.
         const int S = w.split;
         const int R = 128 / S;
         const int d = r / R;                   // rank that reduces this row
@@ -785,6 +796,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         const uint32_t slot_bytes = uint32_t(R * MMA_N * 4);
         const uint32_t stage_row = tiles_base + uint32_t(d) * slot_bytes;
         const uint32_t recv_slots = tiles_base + uint32_t(STAGES * STAGE_BYTES);
+        const uint32_t chunk_bytes = uint32_t(R * 128);
+        // the copy this thread issues (threads 0 .. S-1 other than this CTA's rank)
+        const bool sender = et < S && et != c.s;
+        const uint32_t send_src = tiles_base + uint32_t(et) * slot_bytes;
+        const uint32_t send_dst =
+            sender ? ptx::map_to_rank(recv_slots + uint32_t(c.s < et ? c.s : c.s - 1) * slot_bytes, uint32_t(et)) : 0u;
+        const uint32_t send_bar = sender ? ptx::map_to_rank(ptx::smem_u32(recvbar), uint32_t(et)) : 0u;
 #pragma unroll 1
         for (int c0 = 0; c0 < MMA_N; c0 += 32) {
           uint32_t raw[32];
@@ -793,20 +811,18 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           ptx::tmem_ld_wait();
 #pragma unroll
           for (int j4 = 0; j4 < 8; ++j4)
-            ptx::st_shared_v4(stage_row + part_offset<MMA_N>(rr, c0 / 4 + j4), raw[4 * j4], raw[4 * j4 + 1],
+            ptx::st_shared_v4(stage_row + push_offset(rr, c0 / 4 + j4, R), raw[4 * j4], raw[4 * j4 + 1],
                               raw[4 * j4 + 2], raw[4 * j4 + 3]);
+          ptx::fence_proxy_async_smem();                 // the chunk visible to the bulk copies
+          ptx::named_bar_sync(1, 128);
+          if (sender) {
+            const uint32_t off = uint32_t(c0 / 32) * chunk_bytes;
+            ptx::bulk_copy_to_peer(send_dst + off, send_src + off, chunk_bytes, send_bar);
+          }
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
         released = true;
-        ptx::fence_proxy_async_smem();                   // slices visible to the bulk copies
-        ptx::named_bar_sync(1, 128);
-        if (et < S && et != c.s) {
-          const uint32_t slot = uint32_t(c.s < et ? c.s : c.s - 1);
-          ptx::bulk_copy_to_peer(ptx::map_to_rank(recv_slots + slot * slot_bytes, uint32_t(et)),
-                                 tiles_base + uint32_t(et) * slot_bytes, slot_bytes,
-                                 ptx::map_to_rank(ptx::smem_u32(recvbar), uint32_t(et)));
-        }
         if (first_unit && et == 0) trace_stamp(trace, kTrPartials);
         bool ok2 = ptx::mbar_wait_cluster(ptx::smem_u32(recvbar), 0, abort_flag);
         ok2 = ptx::named_bar_and(1, 128, ok2);
