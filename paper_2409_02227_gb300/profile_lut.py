@@ -211,6 +211,15 @@ class Bench:
         return times[len(times) // 2]
 
 
+def pick_variant(times: Dict[int, Sequence[float]]) -> int:
+    """The variant with the smallest mean, over the sample points, of its time
+    relative to the fastest variant at that point (ties: the smaller id)."""
+    n = len(next(iter(times.values())))
+    fastest = [min(ts[pi] for ts in times.values()) for pi in range(n)]
+    score = {v: sum(t / f for t, f in zip(ts, fastest)) / n for v, ts in times.items()}
+    return min(times, key=lambda v: (score[v], v))
+
+
 def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) -> dict:
     """Steps 1 and 2 for one bucket, at each of its sample points; a variant's
     score is its mean time relative to the fastest candidate at each point,
@@ -226,9 +235,7 @@ def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) 
         for v, ts in times.items():
             for pi, t in enumerate(ts):
                 rows.append(dict(step=step, variant=v, point=pi, us=t, **extra))
-        fastest = [min(ts[pi] for ts in times.values()) for pi in range(len(points))]
-        score = {v: sum(t / f for t, f in zip(ts, fastest)) / len(points) for v, ts in times.items()}
-        v = min(variants, key=lambda x: (score[x], x))
+        v = pick_variant(times)
         return v, times[v]
 
     winners = {}

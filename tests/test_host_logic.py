@@ -111,3 +111,16 @@ def test_corun_flags_rule():
         lut = P.write_lut([((7, 10, 12, 0), 4, [10, 11, 12, 13, 14], flags)], 132, 152)
         conc, v, rc = pr.corun_plan(pr.Desc(128, 1024, 4096, 0), lut, pr.POLICY_AUTO)
         assert conc == 1 and v == (11 if name.startswith("v1") else 10) and rc == int(name.split("rc")[1])
+
+
+def test_pick_variant_scores_relative_times():
+    # one point: the fastest wins
+    assert P.pick_variant({3: [10.0], 7: [9.0], 5: [9.5]}) == 7
+    # two points: 7 is fastest at the first point by 1%, but 40% off at the
+    # second; 3 is 5% off at the first and fastest at the second -> 3
+    assert P.pick_variant({3: [10.5, 20.0], 7: [10.0, 28.0]}) == 3
+    # relative, not absolute: a 1 us point and a 100 us point weigh the same
+    # (mean ratios 1.10 vs 1.15; summed times would pick 2: 121 vs 101.3 us)
+    assert P.pick_variant({1: [1.0, 120.0], 2: [1.3, 100.0]}) == 1
+    # ties -> smaller id
+    assert P.pick_variant({9: [2.0, 4.0], 4: [2.0, 4.0]}) == 4
