@@ -429,3 +429,50 @@ def test_fused_dispatch_matches_strict_groups(cuda_ok, pick):
             if x.dtype == torch.bfloat16:
                 x, y = x.view(torch.int16), y.view(torch.int16)
             assert torch.equal(x, y), f"sweep {j} gemm {i}"
+
+
+def test_phase_trace_regions_per_launch(cuda_ok):
+    # A run of several launches traces into consecutive regions, one per
+    # launch in launch order: each region's CTAs record its grid size and
+    # their index, every CTA stamps its phases in order, and the units over
+    # all regions add up to the plan's units.
+    lut = G.goldy_lut_load(G.DEFAULT_LUT)
+    st = wl.make_sweep_set(_multi_group_sweep_sets(lut, 1)[0])
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    L = Launch(sched, st.a, st.b, [s.out_dtype for s in st.specs])
+    ctas = 8192
+    trace = torch.zeros(ctas * 16, dtype=torch.int64, device="cuda")
+    A_, B_, C_ = L.ptrs()
+    G.goldy_run_ex(sched, A_, B_, C_, L.ws.data_ptr(), L.ws_bytes, [x.cuda_stream for x in L.streams],
+                   trace=trace.data_ptr(), trace_ctas=ctas)
+    L.results()
+    t = trace.view(ctas, 16).cpu()
+    off, regions, units = 0, 0, 0
+    while off < ctas and int(t[off, 12]) > 0:
+        grid = int(t[off, 12])
+        rows = t[off:off + grid]
+        assert (rows[:, 12] == grid).all() and (rows[:, 13] == torch.arange(grid)).all()
+        for r in rows.tolist():
+            # every stamp a CTA wrote lies between its set-up and its exit (the
+            # odd CTA of a pair issues no MMAs and leaves those stamps at 0)
+            assert 0 < r[0] <= r[1] <= r[9]
+            for k in (2, 3, 4, 5, 8):
+                assert r[k] == 0 or r[1] <= r[k] <= r[9], (k, r)
+            assert r[5] <= r[8]
+        units += int(rows[:, 14].sum())
+        off += grid
+        regions += 1
+    assert regions >= 2
+    assert int(t[off:, 0].abs().sum()) == 0                     # nothing written past the last region
+    expect = 0
+    for i in range(len(descs)):
+        _, v, _, _ = G.goldy_schedule_entry(sched, i)
+        info = G.goldy_variant_info_get(v)
+        s = st.specs[i]
+        rows_ = info["mma_n"] if info["swap_ab"] else (256 if info["cta_pair"] == 2 else 128)
+        cols = 128 if info["swap_ab"] else info["mma_n"]
+        tiles = -(-s.M // rows_) * -(-s.N // cols)
+        split = 1 if info["cta_pair"] == 2 else min(info["split_k"], -(-s.K // 64))
+        expect += tiles * split * (2 if info["cta_pair"] == 2 else 1)   # a pair unit counts on both CTAs
+    assert units == expect
