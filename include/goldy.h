@@ -235,7 +235,8 @@ goldy_status goldy_schedule_build(const goldy_gemm_desc* descs, int n, const int
                                   goldy_schedule** out);
 
 /* Sizes of a schedule.  workspace_bytes is the device workspace goldy_run
- * needs (split-K partial tiles and arrival counters, 0 if none). */
+ * needs (split-K partial tiles and arrival counters, and for GOLDY_PLAN_FUSED
+ * schedules of several GEMMs 8 bytes of unit counters per GEMM; 0 if none). */
 goldy_status goldy_schedule_query(const goldy_schedule* s, int* n_gemms, int* n_groups,
                                   int* max_streams, size_t* workspace_bytes);
 
@@ -258,10 +259,10 @@ void goldy_schedule_free(goldy_schedule* s);
  * workspace_bytes (may be null when that is 0), zero-filled by the caller
  * before its first use — the kernels leave it zero-filled after every
  * complete run; streams[0 .. n_streams-1] are CUDA streams with n_streams >=
- * max_streams.  Groups run in order; a group forks from streams[0] and joins
- * back to it, so work queued on streams[0] before the call happens before
- * every GEMM and work queued on streams[0] after it happens after all of
- * them.  Slot k runs on streams[k].  Asynchronous: returns after launching;
+ * max_streams.  Groups run in order (in GOLDY_PLAN_FUSED mode by launch
+ * priority, see there); the run forks from streams[0] and joins back to it,
+ * so work queued on streams[0] before the call happens before every GEMM and
+ * work queued on streams[0] after it happens after all of them.  Slot k runs on streams[k].  Asynchronous: returns after launching;
  * no allocation, no synchronisation.  Errors: GOLDY_ERR_INVALID_ARG (null or
  * misaligned pointers, too few streams, workspace too small),
  * GOLDY_ERR_CUDA (launch failure).  A kernel that gave up a bounded wait

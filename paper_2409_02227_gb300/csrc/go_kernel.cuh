@@ -88,7 +88,14 @@ struct LaunchParams {
   unsigned long long* trace;  // optional phase trace, kTracePerCta stamps per CTA (null: off)
   int32_t cluster;            // 0, or the split-K factor S of every GEMM in the launch when the
                               // launch is made of clusters of S CTAs (the splits of one tile)
+  uint32_t* dyn;              // null: CTA b takes units b, b + grid, ...; else a zeroed pair of
+                              // counters (units taken, CTAs done): after its first unit b a CTA
+                              // takes grid + (counter++), and the last CTA to leave zeroes both
 };
+
+// Units a CTA has taken but its MMA thread and epilogue have not yet both
+// read, at most (a ring of unit indices in shared memory).
+constexpr int kUnitRing = 8;
 
 // Phase trace (optional, for profiling): %globaltimer stamps per CTA.
 enum : int {
@@ -540,11 +547,17 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
   uint64_t* redbar = drain + 1;        // cluster split-K: 2 barriers, alternating by unit
   uint64_t* recvbar = redbar + 2;      // pushed cluster reduction: bytes received
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvbar + 1);
+  uint64_t* ufull = recvbar + 1;       // unit ring: the producer published the unit index
+  uint64_t* uempty = ufull + kUnitRing;  // unit ring: the MMA thread and the epilogue read it
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(uempty + kUnitRing);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
+  volatile int* units_taken = reinterpret_cast<volatile int*>(tmem_slot + 3);
   UnitTable* utab = reinterpret_cast<UnitTable*>(tmem_slot + 4);   // MAXG entries, inside the 1 KB barrier area
-  static_assert((2 * STAGES + 2 * ACC + 4) * 8 + 16 + MAXG * int(sizeof(UnitTable)) <= 1024, "barrier area");
+  volatile int* uring = reinterpret_cast<volatile int*>(utab + MAXG);   // kUnitRing unit indices
+  static_assert((2 * STAGES + 2 * ACC + 4 + 2 * kUnitRing) * 8 + 16 + MAXG * int(sizeof(UnitTable)) +
+                        kUnitRing * 4 <= 1024,
+                "barrier area");
   const int n_gemms = p.n_gemms;
 
   const uint32_t tiles_base = ptx::smem_u32(smem);
@@ -587,8 +600,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       ptx::mbar_init(ptx::smem_u32(&redbar[1]), uint32_t(p.cluster));
     }
     if (push_on) ptx::mbar_init(ptx::smem_u32(recvbar), 1);
+    for (int q = 0; q < kUnitRing; ++q) {
+      ptx::mbar_init(ptx::smem_u32(&ufull[q]), 1);
+      ptx::mbar_init(ptx::smem_u32(&uempty[q]), 2);
+    }
     *abort_flag = 0;
     *last_flag = 0;
+    *units_taken = 0;
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
     // the phase completes once the S - 1 peers' rows of this CTA's slice
@@ -630,7 +648,23 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       int stage = 0;
       uint32_t phase = 0, issued = 0, last_phase = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
+      int u = blockIdx.x, taken = 0;
+      for (int seq = 0; ok; ++seq) {
+        // publish the unit (or the end: an index past the last unit) to the
+        // MMA thread and the epilogue
+        const int slot = seq % kUnitRing;
+        if (seq >= kUnitRing &&
+            !ptx::mbar_wait(ptx::smem_u32(&uempty[slot]), uint32_t((seq / kUnitRing) - 1) & 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        uring[slot] = u;
+        ptx::mbar_arrive(ptx::smem_u32(&ufull[slot]));
+        if (u >= p.total_units) break;
+        ++taken;
+        // the next unit, taken now so that the counter's latency overlaps
+        // this unit's loads
+        const int next = p.dyn ? int(gridDim.x + atomicAdd(p.dyn, 1u)) : u + int(gridDim.x);
         if (issued == 0) trace_stamp(trace, kTrProducerGo);
         const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         const void* ta = &p.tmap_a[c.g];
@@ -667,7 +701,9 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
             phase ^= 1;
           }
         }
+        u = next;
       }
+      *units_taken = taken;
       if (!ok) {
         raise_error(p.err, abort_flag, kErrProducerWait);
         // let every copy this thread started land before the CTA can exit
@@ -681,7 +717,15 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0, acc_used = 0;
       bool ok = true, any = false;
-      for (int u = blockIdx.x; ok && u < p.total_units; u += gridDim.x) {
+      for (int seq = 0; ok; ++seq) {
+        const int slot = seq % kUnitRing;
+        if (!ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        const int u = uring[slot];
+        ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
+        if (u >= p.total_units) break;
         const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         // an accumulator is waited for only once it has been used before
         if ((acc_used >> acc & 1) && !ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
@@ -721,7 +765,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         }
         if (!ok) break;
         ptx::mma_commit(ptx::smem_u32(&tfull[acc]));        // accumulator complete
-        if (u == int(blockIdx.x)) trace_stamp(trace, kTrFirstMmaDone);
+        if (seq == 0) trace_stamp(trace, kTrFirstMmaDone);
         if (++acc == ACC) {
           acc = 0;
           acc_phase ^= 1;
@@ -745,7 +789,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     uint32_t red_it = 0;                    // cluster reductions done by this CTA
     uint32_t stg = 0;                       // staging buffers used (TMA-store epilogue)
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
-    for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
+    for (int seq = 0;; ++seq) {
+      const int slot = seq % kUnitRing;
+      bool okq = ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag);
+      okq = ptx::named_bar_and(1, 128, okq);
+      if (!okq) {
+        if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
+        break;
+      }
+      const int u = uring[slot];
+      if (u >= p.total_units) break;
       const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
       // the GEMM's output description, read from the parameter block while
       // the accumulator is still being computed
@@ -758,8 +811,10 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
         break;
       }
+      // every epilogue thread has read the unit's slot (the barrier above)
+      if (et == 0) ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
       ptx::tc_fence_after();
-      const bool first_unit = (u == int(blockIdx.x));
+      const bool first_unit = (seq == 0);
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
@@ -1003,10 +1058,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   __syncthreads();
   if (threadIdx.x == 0) {
     trace_stamp(trace, kTrEnd);
-    if (trace) {
-      int n = 0;
-      for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) ++n;
-      trace[blockIdx.x * kTracePerCta + kTrUnits] = n;
+    if (trace) trace[blockIdx.x * kTracePerCta + kTrUnits] = *units_taken;
+    if (p.dyn) {
+      // every CTA has stopped taking units once all have counted themselves
+      // out: the last one zeroes the counters for the next launch
+      __threadfence();
+      if (atomicAdd(p.dyn + 1, 1u) == gridDim.x - 1) {
+        p.dyn[0] = 0u;
+        p.dyn[1] = 0u;
+        __threadfence();
+      }
     }
   }
   // no CTA of a cluster leaves while a peer may still signal its barriers

@@ -122,6 +122,9 @@ struct GemmPlan {
   size_t ws_part_off = 0;   // byte offsets into the caller's workspace
   size_t ws_cnt_off = 0;
   size_t ws_bytes = 0;
+  // a fused launch led by this GEMM may hand out its units through a pair of
+  // counters here (fused schedules of several GEMMs; kNoOffset otherwise)
+  size_t ws_dyn_off = ~size_t(0);
 };
 
 struct Group {

@@ -371,6 +371,14 @@ void finalize_schedule(goldy_schedule* s) {
       gp.ws_bytes = off - gp.ws_part_off;
     }
   }
+  // fused schedules of several GEMMs: a pair of unit counters per GEMM (a
+  // fused launch uses its first member's); zero like the split-K counters
+  if ((s->flags & GOLDY_PLAN_FUSED) && s->gemms.size() > 1) {
+    for (size_t i = 0; i < s->gemms.size(); ++i) s->gemms[i].ws_dyn_off = off + 8 * i;
+    off = align(off + 8 * s->gemms.size());
+  } else {
+    for (auto& gp : s->gemms) gp.ws_dyn_off = ~size_t(0);
+  }
   s->workspace_bytes = off;
 }
 

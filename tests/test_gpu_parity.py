@@ -476,3 +476,39 @@ def test_phase_trace_regions_per_launch(cuda_ok):
         split = 1 if info["cta_pair"] == 2 else min(info["split_k"], -(-s.K // 64))
         expect += tiles * split * (2 if info["cta_pair"] == 2 else 1)   # a pair unit counts on both CTAs
     assert units == expect
+
+
+def test_fused_launch_with_unequal_units_hands_them_out_dynamically(cuda_ok):
+    # One fused launch (kind n64_full, split 1, GPU/4 caps: 76 CTAs) over
+    # 64 units of 4 K blocks and 16 units of 32 K blocks: more units than
+    # CTAs and lengths 8x apart, so the units are handed out by the launch's
+    # counter, longest first.  Results match the oracle and, bit for bit, each
+    # GEMM run alone; repeated runs and replays give the same bytes (the last
+    # CTA leaves the counter zeroed: a stale counter would skip units and
+    # leave the NaN fill in C).
+    shapes = [(512, 1024, 256), (256, 512, 2048)]
+    A, B = zip(*[inputs(M, N, K, seed=1100 + i) for i, (M, N, K) in enumerate(shapes)])
+    v = vid(0, 1, 4)
+    alone = [run_explicit([A[i]], [B[i]], [F32], [v])[0] for i in range(2)]
+    descs = [G.desc(M, N, K, F32) for (M, N, K) in shapes]
+    s = G.goldy_schedule_build(descs, [0, 0], [v, v], [0, 1], G.GOLDY_PLAN_FUSED)
+    L = Launch(s, list(A), list(B), [F32, F32])
+    for rep in range(3):
+        for c in L.dC:
+            c.fill_(float("nan"))
+        L.run()
+        got = L.results()
+        for i in range(2):
+            if rep == 0:
+                check_close(got[i], A[i], B[i], f"dynamic units gemm {i}")
+            assert torch.equal(got[i], alone[i]), f"run {rep} gemm {i}"
+    ex = L.exec()
+    for rep in range(3):
+        for c in L.dC:
+            c.fill_(float("nan"))
+        torch.cuda.synchronize()
+        G.goldy_exec_launch(ex)
+        got = L.results()
+        for i in range(2):
+            assert torch.equal(got[i], alone[i]), f"replay {rep} gemm {i}"
+    del ex
