@@ -94,7 +94,9 @@ struct LaunchParams {
 };
 
 // Units a CTA has taken but its MMA thread and epilogue have not yet both
-// read, at most (a ring of unit indices in shared memory).
+// read, at most (a ring of unit indices in shared memory, used when the
+// launch hands units out from a counter; with the static round-robin every
+// role computes the sequence itself).
 constexpr int kUnitRing = 8;
 
 // Phase trace (optional, for profiling): %globaltimer stamps per CTA.
@@ -650,16 +652,18 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       bool ok = true;
       int u = blockIdx.x, taken = 0;
       for (int seq = 0; ok; ++seq) {
-        // publish the unit (or the end: an index past the last unit) to the
-        // MMA thread and the epilogue
-        const int slot = seq % kUnitRing;
-        if (seq >= kUnitRing &&
-            !ptx::mbar_wait(ptx::smem_u32(&uempty[slot]), uint32_t((seq / kUnitRing) - 1) & 1u, abort_flag)) {
-          ok = false;
-          break;
+        if (p.dyn) {
+          // publish the unit (or the end: an index past the last unit) to
+          // the MMA thread and the epilogue
+          const int slot = seq % kUnitRing;
+          if (seq >= kUnitRing &&
+              !ptx::mbar_wait(ptx::smem_u32(&uempty[slot]), uint32_t((seq / kUnitRing) - 1) & 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uring[slot] = u;
+          ptx::mbar_arrive(ptx::smem_u32(&ufull[slot]));
         }
-        uring[slot] = u;
-        ptx::mbar_arrive(ptx::smem_u32(&ufull[slot]));
         if (u >= p.total_units) break;
         ++taken;
         // the next unit, taken now so that the counter's latency overlaps
@@ -718,13 +722,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       uint32_t phase = 0, acc_phase = 0, acc_used = 0;
       bool ok = true, any = false;
       for (int seq = 0; ok; ++seq) {
-        const int slot = seq % kUnitRing;
-        if (!ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag)) {
-          ok = false;
-          break;
+        int u = int(blockIdx.x) + seq * int(gridDim.x);   // static round-robin
+        if (p.dyn) {
+          const int slot = seq % kUnitRing;
+          if (!ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          u = uring[slot];
+          ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
         }
-        const int u = uring[slot];
-        ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
         if (u >= p.total_units) break;
         const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         // an accumulator is waited for only once it has been used before
@@ -791,13 +798,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
     for (int seq = 0;; ++seq) {
       const int slot = seq % kUnitRing;
-      bool okq = ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag);
-      okq = ptx::named_bar_and(1, 128, okq);
-      if (!okq) {
-        if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
-        break;
+      int u = int(blockIdx.x) + seq * int(gridDim.x);     // static round-robin
+      if (p.dyn) {
+        bool okq = ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag);
+        okq = ptx::named_bar_and(1, 128, okq);
+        if (!okq) {
+          if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
+          break;
+        }
+        u = uring[slot];
       }
-      const int u = uring[slot];
       if (u >= p.total_units) break;
       const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
       // the GEMM's output description, read from the parameter block while
@@ -812,7 +822,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         break;
       }
       // every epilogue thread has read the unit's slot (the barrier above)
-      if (et == 0) ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
+      if (p.dyn && et == 0) ptx::mbar_arrive(ptx::smem_u32(&uempty[slot]));
       ptx::tc_fence_after();
       const bool first_unit = (seq == 0);
       if (first_unit && et == 0) trace_stamp(trace, kTrFirstAcc);
