@@ -187,3 +187,20 @@ def test_packaged_tables_and_predictor_load():
     m = open(G.DEFAULT_PREDICTOR, "rb").read()
     G.goldy_predictor_from_memory(m)
     assert P.parse_model(m).sm_count == 152
+
+
+def test_fused_schedules_reserve_unit_counters():
+    # a fused schedule of several GEMMs reserves 8 bytes of unit counters per
+    # GEMM (256-byte aligned) after the split-K regions; other schedules none
+    descs = [G.desc(256, 256, 512), G.desc(128, 512, 256), G.desc(64, 256, 1024)]
+    v = G.variant_id(0, 1, 1)                      # no split-K: no partial regions
+    plain = G.goldy_schedule_build(descs, [0, 0, 0], [v] * 3, [0, 1, 2])
+    fused = G.goldy_schedule_build(descs, [0, 0, 0], [v] * 3, [0, 1, 2], G.GOLDY_PLAN_FUSED)
+    one = G.goldy_schedule_build(descs[:1], [0], [v], [0], G.GOLDY_PLAN_FUSED)
+    assert G.goldy_schedule_query(plain)[3] == 0
+    assert G.goldy_schedule_query(one)[3] == 0
+    assert G.goldy_schedule_query(fused)[3] == 256
+    vs = G.variant_id(0, 2, 1)                     # split 2 on the first GEMM
+    split = G.goldy_schedule_build(descs, [0, 0, 0], [vs, v, v], [0, 1, 2])
+    split_fused = G.goldy_schedule_build(descs, [0, 0, 0], [vs, v, v], [0, 1, 2], G.GOLDY_PLAN_FUSED)
+    assert G.goldy_schedule_query(split_fused)[3] == G.goldy_schedule_query(split)[3] + 256
