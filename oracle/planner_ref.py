@@ -242,7 +242,10 @@ def preferred_cd(speedup: dict, gain: float = 0.05, near: float = 0.01) -> int:
     """Preferred CD from measured speedups over serial execution (Sec. 4.3:
     the CD with the most speedup; Sec. 5.4: sequential unless some CD gains at
     least 5%).  Among CDs whose speedup is within ``near`` (relative) of the
-    best, the largest wins (the paper does not address near-ties).
+    best, the largest wins: Sec. 4.3 names the CD with the most speedup and
+    neither it nor Sec. 5.4 addresses near-ties; with fused waves a larger CD
+    costs no more per GEMM on a near-tie, and a larger preference lets the
+    heterogeneous rule (Sec. 6.6) keep more keys in one group.
     ``speedup[1]`` is 1 by definition."""
     cands = {cd: s for cd, s in speedup.items() if cd in CD_CLASSES and cd != 1}
     if not cands:
