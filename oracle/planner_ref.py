@@ -238,22 +238,22 @@ def serialize(schedule) -> bytes:
     return struct.pack("<%dI" % len(words), *words)
 
 
-def preferred_cd(speedup: dict, gain: float = 0.05, near: float = 0.01) -> int:
-    """Preferred CD from measured speedups over serial execution (Sec. 4.3:
-    the CD with the most speedup; Sec. 5.4: sequential unless some CD gains at
-    least 5%).  Among CDs whose speedup is within ``near`` (relative) of the
-    best, the largest wins: Sec. 4.3 names the CD with the most speedup and
-    neither it nor Sec. 5.4 addresses near-ties; with fused waves a larger CD
-    costs no more per GEMM on a near-tie, and a larger preference lets the
-    heterogeneous rule (Sec. 6.6) keep more keys in one group.
-    ``speedup[1]`` is 1 by definition."""
-    cands = {cd: s for cd, s in speedup.items() if cd in CD_CLASSES and cd != 1}
-    if not cands:
-        return 1
-    best = max(cands.values())
-    if best < 1.0 + gain:
-        return 1
-    return max(cd for cd, s in cands.items() if s >= best * (1.0 - near))
+def preferred_cd(speedup: dict, gain: float = 0.05) -> int:
+    """Preferred CD from measured speedups over serial execution.
+
+    Sec. 4.3 (Dynamic logic for concurrency control): a GEMM's preferred CD
+    is the CD under which it shows the most speedup.  Sec. 5.5
+    (Configurations): the paper's Oracle runs the GEMMs sequentially unless
+    some CD gains at least 5% over sequential.  So: the largest speedup among
+    the CD classes wins; exact ties go to the smaller CD (the paper does not
+    address ties; the smaller CD shares the GPU among fewer GEMMs); CD 1
+    unless that largest speedup reaches 1 + ``gain``.  ``speedup[1]`` is 1
+    by definition."""
+    best_cd, best = 1, 1.0
+    for cd in CD_CLASSES[1:]:
+        if cd in speedup and speedup[cd] > best:
+            best_cd, best = cd, speedup[cd]
+    return best_cd if best >= 1.0 + gain else 1
 
 
 def corun_plan(d: Desc, lut_bytes: bytes, policy: int) -> Tuple[int, int, int]:

@@ -17,9 +17,8 @@ list:
          the GO-Kernel for that CD.  The CD-1 kernel is the whole-GPU winner (the
          isolation-tuned kernel);
   preferred CD: speedup(CD) = CD * T(1) / T(CD) over running the copies one
-         after another; the largest wins, but sequential (CD 1) unless some
-         CD gains at least 5% (Sec. 5.4); CDs within 1% of the best go to the
-         smaller one.
+         after another; the largest wins (exact ties: the smaller CD), but
+         sequential (CD 1) unless some CD gains at least 5% (Sec. 5.5).
 
 Each bucket (floor log2 of M, N, K; output dtype) is profiled at two
 points: its lower edge (M, N, K = powers of two), where DNN layer sizes
@@ -81,21 +80,15 @@ def write_lut(entries, n_variants: int, sm_count: int) -> bytes:
     return bytes(out)
 
 
-def preferred_cd(speedup: Dict[int, float], gain: float = 0.05, near: float = 0.01) -> int:
-    """Largest-speedup CD, sequential unless the gain reaches ``gain``; CDs
-    within ``near`` of the best resolve to the largest (a larger CD costs no
-    more per GEMM on a near-tie, and lets a heterogeneous set run in fewer
-    groups: the planner merges keys only while each prefers the group's size)."""
+def preferred_cd(speedup: Dict[int, float], gain: float = 0.05) -> int:
+    """The CD with the largest speedup over running the copies one after
+    another (Sec. 4.3), exact ties to the smaller CD; sequential (1) unless
+    that speedup reaches 1 + ``gain`` (Sec. 5.5's Oracle configuration)."""
     best_cd, best = 1, 1.0
     for cd in (2, 4, 8, 16):
         if cd in speedup and speedup[cd] > best:
             best_cd, best = cd, speedup[cd]
-    if best < 1.0 + gain:
-        return 1
-    for cd in (16, 8, 4, 2):
-        if cd in speedup and speedup[cd] >= best * (1.0 - near):
-            return cd
-    return best_cd
+    return best_cd if best >= 1.0 + gain else 1
 
 
 def logged_pref(rec: dict) -> int:
@@ -357,6 +350,32 @@ def add_corun_flags(out_dir: str, fused: bool, partition=None) -> None:
     print(f"co-run at once on {sum(1 for e in entries if e[3] & 1)} of {len(entries)} buckets", flush=True)
 
 
+def rebuild_lut(profile_path: str, out_path: str, corun_path: str = None, sm_count: int = 0) -> int:
+    """Re-derive a table from its profiling logs alone (no GPU): each
+    bucket's preferred CD from its logged speedups under the current rule,
+    its kernels as logged, its co-run flags from the logged step-3 times
+    (when a co-run log is given).  The SM count comes from `sm_count` or
+    from the table already at `out_path`.  Returns the number of entries."""
+    recs = {}
+    for line in open(profile_path):
+        r = json.loads(line)
+        recs[tuple(r["key"])] = r
+    flags = {}
+    if corun_path:
+        for line in open(corun_path):
+            r = json.loads(line)
+            flags[tuple(r["key"])] = corun_flags(r["t_us"])
+    if sm_count <= 0:
+        with open(out_path, "rb") as f:
+            sm_count = struct.unpack_from("<I", f.read(32), 20)[0]
+    entries = [(k, logged_pref(r), r["variants"], flags.get(k, 0)) for k, r in recs.items()]
+    lut = write_lut(entries, G.goldy_variant_count(), sm_count)
+    G.goldy_lut_from_memory(lut)          # validate with the library's own parser
+    with open(out_path, "wb") as f:
+        f.write(lut)
+    return len(entries)
+
+
 def profile_dataset_gemm(shape, lut, log, fused: bool = True) -> dict:
     """Training record for the CD predictor (Sec. 4.3): time CD copies of one
     GEMM co-running with the table's GO-Kernel for each CD class (the kernels
@@ -434,6 +453,9 @@ def main(argv=None) -> int:
                     help="buckets of the batched study's B-GEMMs (M x batch rows)")
     ap.add_argument("--corun-flags", action="store_true",
                     help="step 3 over the table already profiled in --out: set each bucket's co-run flag")
+    ap.add_argument("--rebuild", nargs="+", default=None, metavar=("PROFILE_JSONL", "CORUN_JSONL"),
+                    help="no GPU: re-derive the table in --out (a file) from a profile log and, optionally, "
+                         "a co-run log, under the current preferred-CD and co-run rules")
     ap.add_argument("--configs", action="store_true", help="buckets of the fixed workload sets")
     ap.add_argument("--sweep", action="store_true", help="buckets of the 64 randomized sets")
     ap.add_argument("--keys", nargs="*", default=[], help="extra buckets lm,ln,lk,out")
@@ -445,6 +467,10 @@ def main(argv=None) -> int:
         return run_dataset(args.dataset, args.dataset_size, args.lut, args.launch == "fused", args.time_budget)
     if not args.out:
         ap.error("--out is required to build a table")
+    if args.rebuild:
+        n = rebuild_lut(args.rebuild[0], args.out, args.rebuild[1] if len(args.rebuild) > 1 else None)
+        print(f"rebuilt {n} entries in {args.out}", flush=True)
+        return 0
     if args.corun_flags:
         part = G.goldy_partition_create(args.partition, 16) if args.partition is not None else None
         add_corun_flags(args.out, args.launch == "fused", part)

@@ -3,9 +3,8 @@
 Input: the training set recorded by ``profile_lut --dataset`` — per GEMM, the
 co-run time of CD copies at every CD class with the table's GO-Kernel for
 that CD.  Each GEMM is labelled with its preferred CD (largest speedup
-CD * T(1) / T(CD) over running the copies one after another; sequential
-unless some CD gains at least 5%; CDs within 1% of the best go to the
-smaller), and described by the 18 features the library computes
+CD * T(1) / T(CD) over running the copies one after another, exact ties to
+the smaller CD; sequential unless some CD gains at least 5%), and described by the 18 features the library computes
 (goldy_lr_features: M, N, K and, per CD class, the table kernel's CTAs of
 work, CTAs per SM and waves).  As in the paper: min-max normalisation, a
 seeded 90% / 10% train / test split, and a multi-class logistic regression

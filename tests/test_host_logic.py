@@ -21,6 +21,24 @@ def test_preferred_cd_matches_oracle():
             if rng.random() < 0.9:
                 sp[cd] = rng.choice([rng.uniform(0.5, 2.5), rng.uniform(0.98, 1.08)])
         assert P.preferred_cd(sp) == pr.preferred_cd(sp), sp
+    # a CD within 1% of the best does not win: the largest speedup does
+    for sp in ({1: 1.0, 2: 1.20, 4: 1.195}, {1: 1.0, 4: 2.126, 8: 2.111}, {1: 1.0, 8: 1.658, 16: 1.647}):
+        assert P.preferred_cd(sp) == pr.preferred_cd(sp) == max(sp, key=sp.get)
+
+
+def test_table_preferences_follow_the_logged_speedups():
+    """The packaged table's preferred CDs are the rule applied to the
+    speedups its profiling log recorded."""
+    import json
+    import struct
+    data = open(G.DEFAULT_LUT, "rb").read()
+    n = struct.unpack_from("<I", data, 12)[0]
+    prefs = {tuple(data[32 + 16 * i:32 + 16 * i + 4]): data[32 + 16 * i + 4] for i in range(n)}
+    log = os.path.join(os.path.dirname(G.DEFAULT_LUT), "lut_profile.jsonl")
+    for line in open(log):
+        r = json.loads(line)
+        sp = {int(c): v for c, v in r["speedup"].items()}
+        assert prefs[tuple(r["key"])] == pr.preferred_cd(sp), r["key"]
 
 
 def test_lut_writer_matches_oracle_format():

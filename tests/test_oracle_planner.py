@@ -157,13 +157,17 @@ def test_schedule_bytes_by_hand():
 
 
 def test_preferred_cd_rule():
+    # Sec. 4.3: the CD with the most speedup; Sec. 5.5: sequential below a 5% gain
     assert pr.preferred_cd({1: 1.0, 2: 1.04, 4: 1.049}) == 1         # below 5%
-    assert pr.preferred_cd({1: 1.0, 2: 1.05}) == 2
+    assert pr.preferred_cd({1: 1.0, 2: 1.05}) == 2                   # exactly 5%
     assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.105}) == 4         # the best
-    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.195}) == 4         # within 1% of the best -> larger
-    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.18, 8: 1.195}) == 8   # 4 is 1.7% off, 8 within 1%
+    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.195}) == 2         # 4 within 1% of the best: the best wins
+    assert pr.preferred_cd({1: 1.0, 2: 1.20, 4: 1.18, 8: 1.195}) == 2
     assert pr.preferred_cd({1: 1.0, 2: 1.10, 4: 1.20, 8: 1.15}) == 4
+    assert pr.preferred_cd({1: 1.0, 4: 2.126, 8: 2.111, 16: 1.925}) == 4
     assert pr.preferred_cd({1: 1.0, 2: 0.8, 16: 1.9}) == 16
+    assert pr.preferred_cd({1: 1.0, 2: 1.3, 8: 1.3}) == 2            # exact tie: the smaller CD
+    assert pr.preferred_cd({1: 1.0, 2: 0.9, 4: 0.7}) == 1            # concurrency only hurts
     assert pr.preferred_cd({1: 1.0}) == 1
 
 
