@@ -724,7 +724,7 @@ def scaling_lut_path(sm_count: int) -> str:
 
 
 def run_scaling_study(args, local):
-    """GPU-scaling study (Sec. 6.7): each study set (4 equal GEMMs, CD 4) run
+    """GPU-scaling study (Sec. 7.4, Scaling GPUs Configuration): each study set (4 equal GEMMs, CD 4) run
     inside SM partitions of a quarter, half and all of the GPU, under the
     default configuration (isolation-tuned kernels, all GEMMs on their own
     streams), sequential, GOLDYLOC with the table tuned inside that partition,
@@ -802,7 +802,7 @@ def run_scaling_study(args, local):
 
 
 def run_batched_study(args, local):
-    """Heterogeneous strided-batched GEMMs (Sec. 6.6): sets of 2 and 4
+    """Heterogeneous strided-batched GEMMs (Sec. 6.7): sets of 2 and 4
     batched attention GEMMs over variable sequence lengths, under default
     (isolation-tuned kernels, every B-GEMM on its own stream), sequential,
     GO at CD = n, and GOLDYLOC; each configuration at its faster replay,
@@ -854,7 +854,7 @@ def run_batched_study(args, local):
 
 
 def run_corun_study(args, local):
-    """GEMM + element-wise add (Sec. 8.1): each study GEMM co-scheduled with
+    """GEMM + element-wise add (Sec. 7.1): each study GEMM co-scheduled with
     an add over its output size under sequential, default (isolation-tuned
     GEMM kernel and the add at once), GO (CD-2 GO-Kernel and a half-GPU add at
     once) and GOLDYLOC (GO where the table marks co-running as paying, else

@@ -56,7 +56,7 @@ typedef enum goldy_status {
 typedef enum goldy_dtype { GOLDY_BF16 = 0, GOLDY_F32 = 1 } goldy_dtype;
 
 /* One GEMM (Sec. 2.1.2), or a strided batch of equal-sized GEMMs (the
- * paper's B-GEMMs, Sec. 6.6): entry i computes C + i*stride_c = (A +
+ * paper's B-GEMMs, Sec. 6.7): entry i computes C + i*stride_c = (A +
  * i*stride_a)(B + i*stride_b).  Sizes, leading dimensions and strides are in
  * elements.  Supported now: trans_a = trans_b = 0, a = b = GOLDY_BF16, c =
  * BF16 or F32, M, N, K >= 0, lda >= K, ldb >= N, ldc >= N, lda and ldb
@@ -79,9 +79,9 @@ typedef struct goldy_schedule goldy_schedule;
 typedef struct goldy_graph goldy_graph;
 
 /* ---- planning policies (goldy_plan flags) -------------------------------
- * The comparison configurations of Sec. 5.4 through one schedule type:
+ * The comparison configurations of Sec. 5.5 through one schedule type:
  *   AUTO        the dynamic logic: preferred CD from the table, min(CD,
- *               available), heterogeneous grouping (Sec. 4.3, Sec. 6.6)
+ *               available), heterogeneous grouping (Sec. 4.3, Sec. 6.7)
  *   SEQUENTIAL  isolation-tuned kernels one after another ("sequential")
  *   DEFAULT     isolation-tuned kernels, every GEMM at once on its own stream
  *               ("default", the naive all-streams launch)
@@ -330,7 +330,7 @@ void goldy_exec_free(goldy_exec* e);
  * partition, so this also times work inside an SM partition. */
 goldy_status goldy_exec_time(const goldy_exec* const* execs, int n, int warmup, int reps, float* ms_per_rep);
 
-/* ---- a GEMM co-scheduled with a non-GEMM kernel (Sec. 8.1) --------------
+/* ---- a GEMM co-scheduled with a non-GEMM kernel (Sec. 7.1) --------------
  * The paper co-runs a GEMM with an element-wise add of the GEMM's output size
  * (2 kernels at once) and finds concurrency worth restricting for
  * memory-bound GEMMs.  The non-GEMM here is Z = X + Y over n contiguous
@@ -380,7 +380,7 @@ void goldy_corun_free(goldy_corun* c);
 /* The element-wise add alone on one stream (rc_div 1, 2 or 4). */
 goldy_status goldy_ewise_add(const void* X, const void* Y, void* Z, int64_t n, int dtype, int rc_div, void* stream);
 
-/* ---- SM partitions (the paper's CU-partition study, Sec. 6.7) -----------
+/* ---- SM partitions (CU-Partition, Sec. 6.9; GPU-Quarter/Half, Sec. 7.4) -----------
  * A partition is a CUDA green context owning a subset of the GPU's SMs plus
  * n_streams (1 .. GOLDY_MAX_STREAMS) non-blocking streams in it; kernels
  * enqueued on those streams run on the partition's SMs only.  min_sms <= 0

@@ -16,10 +16,10 @@ Contents (each module cites the passage it follows):
 * ``schedule``     — brute-force makespan search over every way of running a
                       small GEMM set as consecutive concurrent groups: the
                       paper's "Oracle" configuration that always picks the
-                      right concurrency degree, sequential included (Sec. 5.4).
+                      right concurrency degree, sequential included (Sec. 5.5).
 * ``planner_ref``  — an independent restatement of the dynamic logic's table
                       lookup (bucketize, preferred CD, min(CD, available),
-                      heterogeneous split; Sec. 4.3 and Sec. 6.6), used to check
+                      heterogeneous split; Sec. 4.3 and Sec. 6.7), used to check
                       the product planner byte for byte.
 
 Parity status: ``gemm`` is pinned (identity, permutation, small-integer

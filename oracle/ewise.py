@@ -1,6 +1,6 @@
 """Element-wise add Z = X + Y — TEST INFRASTRUCTURE ONLY.
 
-The non-GEMM kernel the paper co-schedules with a GEMM (Sec. 8.1).  The
+The non-GEMM kernel the paper co-schedules with a GEMM (Sec. 7.1).  The
 operation is defined at the precision the kernel computes in (the paper
 fixes none): each bf16 input is widened exactly to fp32, the two are added
 with one IEEE-754 binary32 addition (round to nearest, ties to even), and for

@@ -168,7 +168,7 @@ if os.environ.get("GOLDY_ORACLE_THREADS"):
 
 
 def gemm_batched(a_bits: np.ndarray, b_bits: np.ndarray) -> np.ndarray:
-    """A strided batch of GEMMs (Sec. 6.6's B-GEMMs): entry i of the result
+    """A strided batch of GEMMs (Sec. 6.7's B-GEMMs): entry i of the result
     is gemm(a_bits[i], b_bits[i]) for a_bits (batch x M x K) and b_bits
     (batch x K x N)."""
     a_bits = _as_bits(a_bits)

@@ -15,10 +15,10 @@ from the table:
 2. Look the key up.  A key the table lacks takes the stored key nearest in
    L1 distance over the three log2 sizes, a differing output dtype adding 16;
    ties go to the smallest stored key.  (Nearest-neighbour reuse of profiled
-   GEMMs echoes the KNN tuning shortcut, Sec. 7.4.)
+   GEMMs echoes the KNN tuning shortcut, Sec. 7.5.)
 3. The CD actually run is the minimum of the preferred CD and the number of
    GEMMs available (Sec. 4.3).
-4. Two or more distinct keys (heterogeneous GEMMs, Sec. 6.6): the paper runs
+4. Two or more distinct keys (heterogeneous GEMMs, Sec. 6.7): the paper runs
    the whole set at once only if every key prefers at least the set's size,
    and otherwise runs homogeneous groups, each with its own CD.  Generalized
    to any number of keys: one block per key, blocks in decreasing order of
@@ -32,7 +32,7 @@ from the table:
    the smallest CD class (1, 2, 4, 8, 16) not below the group's CD.
 
 Forced policies give the paper's comparison configurations through the same
-schedule type (Sec. 5.4): ``sequential`` (isolation-tuned kernels one after
+schedule type (Sec. 5.5): ``sequential`` (isolation-tuned kernels one after
 another), ``default`` (isolation-tuned kernels, all GEMMs at once on their own
 streams), ``go`` (GO-Kernels, all GEMMs at once) and ``force_cd`` (GO-Kernels
 at a fixed CD).
@@ -166,7 +166,7 @@ class Desc:
     N: int
     K: int
     out_dtype: int
-    batch: int = 1          # strided batch entries (Sec. 6.6's B-GEMMs); bucketed by M * batch rows
+    batch: int = 1          # strided batch entries (Sec. 6.7's B-GEMMs); bucketed by M * batch rows
 
 
 def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
@@ -257,7 +257,7 @@ def preferred_cd(speedup: dict, gain: float = 0.05) -> int:
 
 
 def corun_plan(d: Desc, lut_bytes: bytes, policy: int) -> Tuple[int, int, int]:
-    """A GEMM co-scheduled with an element-wise op over its output (Sec. 8.1):
+    """A GEMM co-scheduled with an element-wise op over its output (Sec. 7.1):
     (concurrent, GEMM variant, grid-cap divisor of the element-wise kernel).
     sequential: isolation-tuned kernel, then the op; default: the
     isolation-tuned kernel and the op (whole GPU) at once; go: the CD-2

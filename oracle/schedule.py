@@ -3,7 +3,7 @@ TEST INFRASTRUCTURE ONLY.
 
 What it computes.  The paper's "Oracle" configuration uses the GO-Kernels and
 always picks the right concurrency degree, sequential execution included
-(Sec. 5.4, Configurations).  For a set of n independent GEMMs, a schedule is
+(Sec. 5.5, Configurations).  For a set of n independent GEMMs, a schedule is
 written here as an ordered split of the set into groups that run one after
 another; the GEMMs inside a group run concurrently, so the group's
 concurrency degree (CD) is its size; each GEMM runs one kernel variant chosen

@@ -1,5 +1,5 @@
 // Element-wise add Z = X + Y: the non-GEMM kernel the paper co-schedules
-// with a GEMM (Sec. 8.1: element-wise adds over the GEMM's output size).
+// with a GEMM (Sec. 7.1: element-wise adds over the GEMM's output size).
 //
 // HBM-bound: every element is read twice and written once.  Persistent
 // grid-stride loop over 16-byte vectors (8 bf16 or 4 fp32 per vector), four

@@ -2,7 +2,7 @@
 //
 // What it computes (Sec. 2.1.2): C = A * B for A (M x K, row-major), B
 // (K x N, row-major), fp32 accumulation, fp32 or bf16 (round-to-nearest-even)
-// output; a strided-batched GEMM (Sec. 6.6's B-GEMMs) is `batch` such
+// output; a strided-batched GEMM (Sec. 6.7's B-GEMMs) is `batch` such
 // products at fixed strides, its tiles numbered batch entry by batch entry.
 // Several GEMMs may share one launch (the launch's "units" are the
 // concatenation of their tiles).

@@ -7,7 +7,7 @@
 // processor, so this runs on the host right before launch: integer work over
 // at most 64 descriptors, no CUDA call, a pure function of its inputs.
 //
-// Rules (Sec. 4.3: CD = min(preferred CD, GEMMs available); Sec. 6.6: a
+// Rules (Sec. 4.3: CD = min(preferred CD, GEMMs available); Sec. 6.7: a
 // heterogeneous set runs at once only when every distinct GEMM prefers that
 // many, otherwise homogeneous groups each with its own CD):
 //   key      = (floor log2 M, floor log2 N, floor log2 K, C dtype)
@@ -642,7 +642,7 @@ extern "C" goldy_status goldy_variant_info_get(int id, goldy_variant_info* out) 
 }
 
 // ---------------------------------------------------------------------------
-// A GEMM co-scheduled with an element-wise add (Sec. 8.1)
+// A GEMM co-scheduled with an element-wise add (Sec. 7.1)
 // ---------------------------------------------------------------------------
 extern "C" goldy_status goldy_corun_plan(const goldy_gemm_desc* gemm, const goldy_ewise_desc* ew,
                                          const goldy_lut* lut, int policy, goldy_corun** out) {

@@ -260,7 +260,7 @@ CORUN_CONFIGS = [(f"v{vi}_rc{1 << ri}", 1 | (vi << 1) | (ri << 2)) for vi in (0,
 
 
 def corun_times(bench: "Bench", variants: Sequence[int], target_us: float = 2000.0) -> Dict[str, float]:
-    """Step 3 (Sec. 8.1): the bucket's GEMM with an element-wise add of its
+    """Step 3 (Sec. 7.1): the bucket's GEMM with an element-wise add of its
     output size, one after the other ("sequential": the CD-1 kernel, then the
     add over the whole GPU) and at once in every configuration the table can
     record: the CD-1 or the CD-2 GO-Kernel ("v0", "v1") with the add's grid
@@ -297,7 +297,7 @@ def corun_times(bench: "Bench", variants: Sequence[int], target_us: float = 2000
 
 def corun_flags(t: Dict[str, float], gain: float = 0.05) -> int:
     """The table's co-run flags from step 3's times, with the preferred-CD
-    rule's 5% threshold (Sec. 5.4) applied twice: a configuration other than
+    rule's 5% threshold (Sec. 5.5) applied twice: a configuration other than
     the default one (CD-1 kernel, add over the whole GPU) is recorded only
     when it beats the default by `gain`, and running at once at all only when
     the chosen configuration beats one after the other by `gain` (0:

@@ -15,7 +15,7 @@ Fit: minimise sum_i CE_i + ||W||^2 / (2 C) over W (5 x 18) and the biases b
 gradient.  C is picked by 5-fold cross-validation on the training part.
 
 Evaluation on the held-out part, for 2, 4, 8 and 16 GEMMs available (the
-paper reports accuracy that way, Sec. 6.5): a prediction p counts as right
+paper reports accuracy that way, Sec. 6.6): a prediction p counts as right
 when min(p, n) is the best CD among the classes <= n; the regret is the time
 per GEMM at the chosen CD over the best, against the table's preferred CD
 for the same GEMMs as the baseline.

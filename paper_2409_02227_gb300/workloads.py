@@ -218,7 +218,7 @@ def make_scaling_set(i: int, copies: int = 4) -> GemmSet:
 
 def batched_study_specs(i: int, members: int) -> Tuple[int, List[GemmSpec]]:
     """Set i of the batched study: `members` (2 or 4) heterogeneous strided
-    batched GEMMs of attention over variable-length inputs (Sec. 6.6's
+    batched GEMMs of attention over variable-length inputs (Sec. 6.7's
     B-GEMMs): per member a sequence length L from {128, ..., 2048} and 16 or
     32 heads of dimension 128, as scores = Q K^T (M = L, N = L, K = 128) or
     output = P V (M = L, N = 128, K = L), batch = heads; bf16 out,

@@ -1,4 +1,4 @@
-"""Strided-batched GEMMs (Sec. 6.6's B-GEMMs) on the GPU: every entry of a
+"""Strided-batched GEMMs (Sec. 6.7's B-GEMMs) on the GPU: every entry of a
 batch matches the oracle under every kernel kind, with split-K (cluster and
 last-arriver reductions), fused launches mixing batched and plain GEMMs,
 non-packed strides (the gaps between entries stay untouched), K = 0, and

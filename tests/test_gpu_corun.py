@@ -1,4 +1,4 @@
-"""A GEMM co-scheduled with an element-wise add (Sec. 8.1) on the GPU: under
+"""A GEMM co-scheduled with an element-wise add (Sec. 7.1) on the GPU: under
 every policy the GEMM matches the oracle and the add matches the oracle bit
 for bit (both take the same IEEE fp32 addition and bf16 rounding), over
 ragged lengths, unaligned operands (scalar path), n = 0, and through a

@@ -1,4 +1,4 @@
-"""SM partitions (green contexts): the paper's CU-partition study (Sec. 6.7)
+"""SM partitions (green contexts): the paper's CU-partition study (Sec. 6.9, GOLDYLOC with Resource Partitioning)
 runs the whole method inside a quarter, half or all of the GPU.  Schedules
 run on a partition's streams give the oracle's results, stay on the
 partition's SMs (the per-CTA trace records the SM of every CTA), and a

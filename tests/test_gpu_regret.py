@@ -1,4 +1,4 @@
-"""The dynamic logic against the paper's "Oracle" configuration (Sec. 5.4:
+"""The dynamic logic against the paper's "Oracle" configuration (Sec. 5.5:
 always the right concurrency degree, sequential included), made exhaustive.
 
 For small sets the time of every subset run as one concurrent (fused) group,

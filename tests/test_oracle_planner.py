@@ -1,7 +1,7 @@
 """Pins for the reference planner (CPU only): hand-solved cases of the rules
 it restates — min(preferred CD, available) (Sec. 4.3), the heterogeneous
-all-or-homogeneous-groups rule (Sec. 6.6), the >= 5% sequential rule
-(Sec. 5.4) — plus the LUT and schedule byte formats written out by hand."""
+all-or-homogeneous-groups rule (Sec. 6.7), the >= 5% sequential rule
+(Sec. 5.5) — plus the LUT and schedule byte formats written out by hand."""
 import struct
 
 import pytest
@@ -58,7 +58,7 @@ def test_all_prefer_sequential():
 
 
 def test_heterogeneous_pair_paper_rule():
-    # 8 + 8 GEMMs of two shapes (Sec. 6.6): both prefer 16 -> all 16 at once
+    # 8 + 8 GEMMs of two shapes (Sec. 6.7): both prefer 16 -> all 16 at once
     L = lut((K_SMALL, 16, V_SMALL), (K_BIG, 16, V_BIG))
     descs = [D(512, 1024, 1024)] * 8 + [D(2048, 8192, 2048)] * 8
     groups, per, ms, _ = pr.plan(descs, L)
