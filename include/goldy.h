@@ -420,20 +420,23 @@ void goldy_graph_free(goldy_graph* g);
 /* One GEMM with GO-Kernel variant `variant`, for callers that cannot allocate
  * device memory (the paper has no counterpart; this is a service of this
  * library).  goldy_run needs a caller workspace for split-K variants; callers
- * running inside an open stream capture, under a fixed memory budget, inside a
- * framework that owns all device allocations, or on paths where cudaMalloc's
- * implicit synchronisation is unacceptable cannot provide one.  Here the
- * split-K scratch is a fixed 32 MiB device array compiled into the library
- * (one per GPU that loads it, held until exit); nothing is allocated.
- * Launches on `stream` (cudaStream_t as void*, may be null) and returns
- * without synchronising.  A, B, C, desc: as for goldy_run (16-byte aligned A
- * and B).  Errors: GOLDY_ERR_INVALID_ARG for a bad descriptor, variant or
- * pointer, or when the GEMM would need more than the 32 MiB scratch (the
- * message gives the size); GOLDY_ERR_CUDA for a failed launch.  The first call
- * on a device looks up the scratch's device address (cudaGetSymbolAddress,
- * which may load device code): make it before any stream capture.  All calls
- * share the scratch: calls whose kernels overlap on the GPU race and give
- * wrong results, so serialise them (one stream, or events). */
+ * held to a fixed memory budget, plugins inside a framework that owns all
+ * device allocations, and paths where cudaMalloc's implicit synchronisation
+ * is unacceptable cannot provide one.  Here the split-K scratch is a fixed
+ * 32 MiB device array compiled into the library (one per GPU that loads it,
+ * held until exit); nothing is allocated.  Launches on `stream`
+ * (cudaStream_t as void*, may be null; a stream of an SM partition runs the
+ * GEMM inside the partition, as goldy_run does) and returns without
+ * synchronising.  A, B, C, desc: as for goldy_run (16-byte aligned A and B).
+ * Errors: GOLDY_ERR_INVALID_ARG for a bad descriptor, variant or pointer, or
+ * when the GEMM would need more than the 32 MiB scratch (the message gives the
+ * size); GOLDY_ERR_CUDA for a failed launch.  The first call on a device looks
+ * up the scratch's device address (cudaGetSymbolAddress, which may load
+ * device code) and keeps it for the life of the process: make that call
+ * before any stream capture, and do not call this entry point on a device
+ * after cudaDeviceReset.  All calls share the scratch: calls whose kernels
+ * overlap on the GPU race and give wrong results, so serialise them (one
+ * stream, or events). */
 goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int variant, const void* A,
                                 const void* B, void* C, void* stream);
 

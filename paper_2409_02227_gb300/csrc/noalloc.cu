@@ -3,13 +3,13 @@
 //
 // Split-K GO-Kernels need scratch memory for their partial tiles and arrival
 // counters; goldy_run takes it from a caller-supplied workspace.  Some callers
-// cannot provide one because they cannot allocate device memory where they
-// run GEMMs: code that runs while a CUDA stream capture is open (allocation is
-// not a capturable operation), runtimes that give a kernel library a fixed
-// memory budget and forbid further device allocations, plugins inside a host
+// cannot provide one because they are not allowed to allocate device memory
+// where they run GEMMs: runtimes that give a kernel library a fixed memory
+// budget and forbid further device allocations, plugins inside a host
 // framework that owns every device allocation, and latency-critical paths
-// where cudaMalloc's implicit synchronisation is not acceptable.  For them this
-// entry point keeps the scratch in a fixed array compiled into the library.
+// where cudaMalloc's implicit synchronisation is not acceptable.  For them
+// this entry point keeps the scratch in a fixed array compiled into the
+// library.
 //
 // The array, g_noalloc_scratch, holds kNoAllocScratchBytes (32 MiB).  Every
 // GPU that loads this library's device code holds one copy until the process
@@ -19,14 +19,19 @@
 // In host code `g_noalloc_scratch` is only a host-side stand-in for the device
 // array, not a device address: the device address is looked up once per
 // device with cudaGetSymbolAddress, with that device current, during the first
-// call made on it.  That first call may load this library's device module, so
-// make it before any stream capture begins.
+// call made on it, and kept for the life of the process.  That first call may
+// load this library's device module, so make it before any stream capture
+// begins.  Do not use this entry point on a device after cudaDeviceReset: the
+// module is reloaded and the kept address is no longer valid.
 //
 // Every call shares the one array and leaves the last call's contents in it.
 // The arrival counters are cleared on the caller's stream before each launch;
 // the partial tiles need no clearing (each split writes its whole tile before
 // any split reads it).  Calls whose kernels overlap on the GPU (other streams,
 // other host threads) race on the array and give wrong results: serialise them.
+//
+// A stream of an SM partition (goldy_partition_query) runs the GEMM inside
+// the partition, as goldy_run does.
 //
 // Nothing here calls cudaMalloc, cudaFree or any allocating library routine.
 #include <cuda_runtime.h>
@@ -44,7 +49,7 @@ constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 goldy_status launch_planned_gemm(const GemmPlan& gp, const void* A, const void* B, void* C, unsigned char* ws,
-                                 void* stream);
+                                 void* stream, size_t clear_off, size_t clear_bytes);
 
 namespace {
 constexpr int kMaxDevices = 64;
@@ -115,15 +120,14 @@ extern "C" goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int vari
   unsigned char* scratch = nullptr;
   st = noalloc_scratch(&scratch);
   if (st != GOLDY_OK) return st;
+  size_t clear_bytes = 0;
   if (need > 0) {
     gp.ws_part_off = 0;
     gp.ws_cnt_off = cnt_off;
     gp.ws_bytes = need;
-    cudaError_t e = cudaMemsetAsync(scratch + cnt_off, 0, size_t(tiles) * sizeof(uint32_t),
-                                    static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return fail(GOLDY_ERR_CUDA, std::string("cudaMemsetAsync (counters): ") + cudaGetErrorString(e));
+    clear_bytes = size_t(tiles) * sizeof(uint32_t);
   }
-  st = launch_planned_gemm(gp, A, B, C, scratch, stream);
+  st = launch_planned_gemm(gp, A, B, C, scratch, stream, cnt_off, clear_bytes);
   if (st != GOLDY_OK) return st;
   return ok();
 }

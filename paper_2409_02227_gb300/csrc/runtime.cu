@@ -1350,13 +1350,23 @@ extern "C" goldy_status goldy_device_info(int variant_id, int* sm_count, int* ct
 
 namespace goldy {
 // Launch one GEMM whose plan fields (kind, tiles, split, workspace offsets)
-// are already filled in, with `ws` as the workspace base.  Shares the
-// per-device setup and the launch code of goldy_run.
+// are already filled in, with `ws` as the workspace base, after zeroing
+// `clear_bytes` bytes of it at `clear_off` on the same stream.  Shares the
+// per-device setup and the launch code of goldy_run, and like goldy_run runs
+// inside the SM partition `stream` belongs to (its green context current,
+// grid caps from its SM count).
 goldy_status launch_planned_gemm(const GemmPlan& gp, const void* A, const void* B, void* C, unsigned char* ws,
-                                 void* stream) {
+                                 void* stream, size_t clear_off, size_t clear_bytes) {
   DeviceState* d = nullptr;
   goldy_status st = device_state(&d);
   if (st != GOLDY_OK) return st;
+  PartitionScope part;
+  st = part.enter(stream);
+  if (st != GOLDY_OK) return st;
+  if (clear_bytes > 0) {
+    cudaError_t e = cudaMemsetAsync(ws + clear_off, 0, clear_bytes, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync (split-K counters)");
+  }
   return launch_gemm(*d, gp, A, B, C, ws, static_cast<cudaStream_t>(stream));
 }
 }  // namespace goldy

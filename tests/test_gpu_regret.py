@@ -8,8 +8,9 @@ split into consecutive groups under those times, and the planner's own
 schedule is timed directly.  The regret (planner / best - 1) must stay small;
 the paper reports its predictor within 3% geomean of its Oracle.  The plan
 with the trained logistic-regression predictor (Eq. 1) is timed the same way.
-Results are
-also written to gpurun_out/regret.json when that folder exists."""
+Each set's
+record is also appended, as one JSON line, to the file named by the
+environment variable GOLDY_REGRET_LOG when it is set."""
 import json
 import math
 import os
@@ -101,9 +102,9 @@ def test_planner_regret_vs_exhaustive_oracle(cuda_ok, name):
               "oracle_partition": [list(b) for b in best.partition],
               "planner_groups": [e[0] for e in entries_plan],
               "subset_us": {",".join(map(str, k)): v for k, v in cache.items()}}
-    out = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "gpurun_out")
-    if os.path.isdir(out):
-        with open(os.path.join(out, "regret.jsonl"), "a") as f:
+    log = os.environ.get("GOLDY_REGRET_LOG")
+    if log:
+        with open(log, "a") as f:
             f.write(json.dumps(record) + "\n")
     assert math.isfinite(regret)
     assert regret < 0.35, record
