@@ -5,9 +5,11 @@ One step = one pass of the whole hot path over one synthetic GEMM set: the
 dynamic logic's plan (computed once; it is a pure function of the shapes)
 replayed as a prepared run of GO-Kernel launches on CD streams (recorded
 once, replayed with plain launches; ``--replay graph`` replays a captured
-CUDA graph instead).  Default
-workload: the tensor-sliced Transformer FFN at low batch, 4 independent
-GEMMs of M=128, N=1024, K=4096, bf16 in, fp32 accumulate, bf16 out.
+CUDA graph instead).  Default workload: the heterogeneous pair of two
+co-running models, 3 GEMMs of M=512, N=1024, K=1024 plus one of M=2048,
+N=8192, K=2048, bf16 in, fp32 accumulate and out — the largest fixed set and
+the compute-bound one.  The other fixed sets are measured on the same line
+as extra keys.
 
 Prints ONE JSON line (rank 0): TFLOP/s of the whole job (all ranks), the
 makespan, speedups over sequential and naive all-streams execution of the
@@ -51,8 +53,10 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=20000)
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["goldy", "reference"], default="goldy")
-    ap.add_argument("--config", default="ffn_slices",
-                    choices=["pair_256", "ffn_slices", "lstm_gates", "hetero_pair"])
+    ap.add_argument("--config", default="hetero_pair",
+                    help="workload: pair_256, ffn_slices, lstm_gates, hetero_pair or sweep_00 .. sweep_63")
+    ap.add_argument("--extra-configs", default="pair_256,ffn_slices,lstm_gates",
+                    help="comma-separated fixed sets also measured on the line ('' for none)")
     ap.add_argument("--lut", default=None, help="lookup table (default: the packaged one)")
     ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
                     help="fused: a wave's same-kind GEMMs share one launch; streams: one launch per GEMM")
@@ -60,6 +64,9 @@ def parse_args(argv=None):
                     help="how the prepared step is replayed: recorded plain launches or a CUDA graph")
     ap.add_argument("--serial-launch", action="store_true",
                     help="plain serialised launches (no overlap of a launch's set-up with the previous kernel)")
+    ap.add_argument("--no-inputs-ready", action="store_true",
+                    help="do not let a launch's loads and MMAs start during the previous kernel's tail "
+                         "(goldy_run_opts.inputs_ready = 0)")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--batched-study", default=None, metavar="FILE",
@@ -210,6 +217,14 @@ def workload_label(specs) -> str:
     return " + ".join(f"{n}x(M={m},N={nn},K={k},{o} out)" for (m, nn, k, o), n in c.items())
 
 
+def load_set(name: str):
+    """A fixed workload set by name, or randomized set j as sweep_jj."""
+    from paper_2409_02227_gb300 import workloads as wl
+    if name.startswith("sweep_"):
+        return wl.make_sweep_set(int(name.split("_")[1]))
+    return wl.make_config(name)
+
+
 # ----------------------------------------------------------------------------- CPU oracle
 def oracle_sample(st, budget_s: float):
     """Run the fp64 oracle over GEMMs of the set (whole GEMMs, in order,
@@ -237,8 +252,7 @@ def run_reference(args, world, rank):
     if rank != 0:
         return 0
     from oracle import gemm as og
-    from paper_2409_02227_gb300 import workloads as wl
-    st = wl.make_config(args.config)
+    st = load_set(args.config)
     # each step computes a fixed number of output entries of every GEMM of the
     # set (exact fp64 dot products), sized so the whole run takes about a minute
     import numpy as np
@@ -288,9 +302,11 @@ def c_shape(s):
 class SetRunner:
     """R rotating device copies of one GEMM set, each with its run prepared
     once: a recorded prepared run (``replay="exec"``, plain launches) or a
-    captured CUDA graph (``replay="graph"``)."""
+    captured CUDA graph (``replay="graph"``).  Construction replays every
+    prepared run once (untimed), so none is first launched inside a timed
+    region."""
 
-    def __init__(self, st, sched, copies, with_events=False, replay="exec", serial_launch=False):
+    def __init__(self, st, sched, copies, with_events=False, replay="exec", serial_launch=False, inputs_ready=True):
         import torch
         from paper_2409_02227_gb300 import goldy as G
         self.G = G
@@ -326,14 +342,21 @@ class SetRunner:
                 torch.cuda.synchronize()
                 evs = {"ev_begin": [e.cuda_event for e in eb], "ev_end": [e.cuda_event for e in ee]}
                 self.events.append((eb, ee))
+            # inputs_ready: no kernel of the run writes an A or B (each step
+            # reads its own copy, written once before any step), so the load
+            # and MMA roles may start during the previous kernel's tail
             if replay == "exec":
                 r = G.goldy_exec_create(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp, serial_launch=serial_launch,
-                                        **evs)
+                                        inputs_ready=inputs_ready, **evs)
             else:
                 r = G.goldy_graph_create_ex(sched, *ptrs, self.ws.data_ptr(), ws_bytes, sp,
-                                            evs.get("ev_begin"), evs.get("ev_end"), serial_launch=serial_launch)
+                                            evs.get("ev_begin"), evs.get("ev_end"), serial_launch=serial_launch,
+                                            inputs_ready=inputs_ready)
             self.runs.append(r)
         self.main = self.streams[0]
+        for k in range(len(self.runs)):
+            self.launch(k)
+        torch.cuda.synchronize()
 
     def __del__(self):
         # destroy the prepared runs before the buffers they read and write
@@ -346,27 +369,52 @@ class SetRunner:
         else:
             self.G.goldy_graph_launch(r, self.main.cuda_stream)
 
-    def timed(self, steps, step_events=0):
-        """Elapsed ms of `steps` back-to-back replays; with `step_events`, the
-        last that many replays are also bracketed by their own event pair on
-        the launching stream (returned as a list of ms)."""
+    def spin(self, us):
+        """Keep the launching stream busy for about `us` microseconds (a
+        clock-cycle spin kernel) so that the host has queued what follows
+        before the GPU reaches it: a timed region then measures the device,
+        not the host's launch rate."""
         torch = self.torch
-        step_events = min(step_events, steps)
-        pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                 for _ in range(step_events)]
-        first = steps - step_events
+        with torch.cuda.stream(self.main):
+            torch.cuda._sleep(int(us * 2000))
+
+    def timed(self, steps, spin_us=200.0):
+        """Elapsed ms of `steps` back-to-back replays (copy k % R for step k),
+        bracketed by one event pair on the launching stream and nothing in
+        between."""
+        torch = self.torch
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        self.spin(spin_us)
         e0.record(self.main)
         for k in range(steps):
-            if k >= first:
-                pairs[k - first][0].record(self.main)
-                self.launch(k)
-                pairs[k - first][1].record(self.main)
-            else:
-                self.launch(k)
+            self.launch(k)
         e1.record(self.main)
         torch.cuda.synchronize()
-        return e0.elapsed_time(e1), [a.elapsed_time(b) for a, b in pairs]
+        return e0.elapsed_time(e1)
+
+    def step_distribution(self, reps, mode, flush=None, spin_us=25.0):
+        """Per-step device time over `reps` single steps, each bracketed by its
+        own event pair: ``cold`` flushes the L2 (writes `flush`, a buffer of
+        twice its size) and rotates the copies before each step; ``warm``
+        replays copy 0 untimed right before each timed replay of copy 0, so
+        its operands sit in the L2.  A short spin before each timed step lets
+        the host queue the step first.  Median, p10 and p90 in us."""
+        torch = self.torch
+        pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for i, (a, b) in enumerate(pairs):
+            if mode == "cold":
+                with torch.cuda.stream(self.main):
+                    flush.zero_()
+                k = i
+            else:
+                self.launch(0)
+                k = 0
+            self.spin(spin_us)
+            a.record(self.main)
+            self.launch(k)
+            b.record(self.main)
+        torch.cuda.synchronize()
+        return percentiles([a.elapsed_time(b) * 1e3 for a, b in pairs])
 
     def launch_durations_ms(self):
         out = []
@@ -376,7 +424,13 @@ class SetRunner:
         return out
 
 
-def time_schedule(st, sched, copies, steps, warm=10):
+def percentiles(xs):
+    xs = sorted(xs)
+    q = lambda f: xs[min(len(xs) - 1, max(0, int(round(f * (len(xs) - 1)))))]
+    return {"median_us": q(0.5), "p10_us": q(0.1), "p90_us": q(0.9), "reps": len(xs)}
+
+
+def time_schedule(st, sched, copies, steps):
     """Makespan (us) of one schedule, replayed both ways (recorded plain
     launches and a CUDA graph); each configuration is credited with its
     faster replay, so that no baseline is slowed by a launch mode that does
@@ -385,52 +439,75 @@ def time_schedule(st, sched, copies, steps, warm=10):
     out = {}
     for mode in ("exec", "graph"):
         r = SetRunner(st, sched, copies, replay=mode)
-        for k in range(warm):
+        for k in range(10):
             r.launch(k)
         torch.cuda.synchronize()
-        out[mode] = r.timed(steps)[0] / steps * 1e3
+        out[mode] = r.timed(steps) / steps * 1e3
         del r
     return min(out.values()), out
 
 
 def cublas_reference_ms(st, copies, steps):
-    """torch.matmul (cuBLAS) for the same set, back to back on one stream: one
-    CUDA graph runs the set once per rotating copy (so the inputs come from
-    HBM), replayed; ms per set.  A reference point only."""
+    """torch.matmul (cuBLAS) for the same set, as a reference point only:
+    ``sequential`` runs the set's GEMMs back to back on one stream;
+    ``streams`` forks one stream per GEMM from the launching stream and joins
+    them back (the naive all-streams launch).  Each is one CUDA graph that
+    runs the set once per rotating copy (so the inputs come from HBM),
+    replayed; ms per set."""
     import torch
     base_a = [a.cuda() for a in st.a]
     base_b = [b.cuda() for b in st.b]
     s = torch.cuda.Stream()
-    keep = []                   # the captured graph reads every copy: keep them all alive
+    side = [torch.cuda.Stream() for _ in st.a]
+    keep = []                   # the captured graphs read every copy: keep them all alive
     for r in range(copies):
         A = base_a if r == 0 else [a.clone() for a in base_a]
         B = base_b if r == 0 else [b.clone() for b in base_b]
         keep.append((A, B))
-    with torch.cuda.stream(s):
-        for a, b in zip(*keep[0]):
-            torch.matmul(a, b)      # warm cuBLAS handles outside the capture
+    for st_ in [s] + side:
+        with torch.cuda.stream(st_):
+            for a, b in zip(*keep[0]):
+                torch.matmul(a, b)      # warm cuBLAS handles on every stream outside the capture
     torch.cuda.synchronize()
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=s):
-        outs = [[torch.matmul(a, b) for a, b in zip(A, B)] for A, B in keep]
-    for _ in range(3):
-        g.replay()
-    torch.cuda.synchronize()
-    reps = max(3, steps // copies)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(reps):
-        g.replay()
-    e1.record()
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / (reps * copies)
-    del g, outs, keep
-    return ms
+    out = {}
+    for mode in ("sequential", "streams"):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            outs = []
+            for A, B in keep:
+                if mode == "sequential":
+                    outs.append([torch.matmul(a, b) for a, b in zip(A, B)])
+                    continue
+                for x in side:
+                    x.wait_stream(s)
+                row = []
+                for x, a, b in zip(side, A, B):
+                    with torch.cuda.stream(x):
+                        row.append(torch.matmul(a, b))
+                for x in side:
+                    s.wait_stream(x)
+                outs.append(row)
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        reps = max(3, steps // copies)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        out[mode] = e0.elapsed_time(e1) / (reps * copies)
+        del g, outs
+    del keep
+    return out
 
 
 def e2e_measure(st, sched, steps):
     """Same metric through host buffers: each step copies A, B from pinned
-    host memory, runs the schedule, and reads C back to pinned host memory."""
+    host memory, runs the schedule, and reads C back to pinned host memory.
+    Also times the copies alone (the same bytes, same streams, no GEMMs):
+    the ceiling the end-to-end number can reach on this host link."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
     _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
@@ -449,28 +526,102 @@ def e2e_measure(st, sched, steps):
     C = [c.data_ptr() for c in dC]
     sp = [s.cuda_stream for s in streams]
 
-    def step():
+    def step(gemm=True):
         with torch.cuda.stream(main):
             for d, h in zip(dA + dB, hA + hB):
                 d.copy_(h, non_blocking=True)
-        G.goldy_run(sched, A, B, C, ws.data_ptr(), ws_bytes, sp)
+        if gemm:
+            G.goldy_run(sched, A, B, C, ws.data_ptr(), ws_bytes, sp)
         with torch.cuda.stream(main):
             for h, d in zip(hC, dC):
                 h.copy_(d, non_blocking=True)
 
-    for _ in range(3):
-        step()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(main)
-    for _ in range(steps):
-        step()
-    e1.record(main)
-    torch.cuda.synchronize()
-    ms_step = e0.elapsed_time(e1) / steps
+    def run(gemm):
+        for _ in range(3):
+            step(gemm)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(main)
+        for _ in range(steps):
+            step(gemm)
+        e1.record(main)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps
+
+    ms_step = run(True)
+    ms_copies = run(False)
     h2d = sum(a.numel() * a.element_size() for a in hA + hB)
     d2h = sum(c.numel() * c.element_size() for c in hC)
-    return ms_step, h2d, d2h
+    return ms_step, ms_copies, h2d, d2h
+
+
+def plan_set(G, st, lut, launch_flag):
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
+    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | launch_flag)
+    plan = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
+    kinds = {(G.goldy_variant_info_get(v)["kind"], st.specs[i].out_dtype) for i, (_, v, _, _) in enumerate(plan)}
+    n_groups = G.goldy_schedule_query(sched)[1]
+    single = bool(launch_flag) and n_groups == 1 and len(kinds) == 1 and plan[0][3] >= len(descs)
+    return descs, sched, plan, single
+
+
+def rotating_copies(st, l2):
+    in_bytes = sum(s.batch * (2 * s.M * s.K + 2 * s.K * s.N) for s in st.specs)
+    return max(2, math.ceil(2 * l2 / in_bytes)), in_bytes
+
+
+def compare_policies(G, st, descs, lut, copies, csteps, launch_flag):
+    comp, modes = {}, {}
+    for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
+                        ("go_all_concurrent", G.GOLDY_PLAN_GO),
+                        ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
+                        ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
+        s2 = G.goldy_plan(descs, lut, flags)
+        comp[name], modes[name] = time_schedule(st, s2, copies, csteps)
+    a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
+    cb = cublas_reference_ms(st, copies, csteps)
+    out = {"comparisons_us": {**comp, "cublas_sequential_reference": cb["sequential"] * 1e3,
+                              "cublas_streams_reference": cb["streams"] * 1e3, "by_replay": modes,
+                              "note": "each configuration at its faster replay (recorded launches or graph); "
+                                      "cuBLAS (torch.matmul) is a reference point only"},
+           "speedup_vs_sequential": comp["sequential"] / a_us,
+           "speedup_vs_naive_streams": comp["naive_streams"] / a_us}
+    return out
+
+
+def roof_of(st, us, hbm, tf_burst, tf_sust):
+    roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
+    bound = "tensor" if st.flops / st.bytes > tf_burst * 1e12 / (hbm * 1e9) else "hbm"
+    out = {"bound": bound, "set_roof_us": roof_us, "frac": roof_us / us}
+    if bound == "tensor":
+        out["frac_sustained"] = st.flops / (tf_sust * 1e12) * 1e6 / us
+    return out
+
+
+def measure_extra(G, name, lut, l2, launch_flag, flush, steps, peaks_):
+    """One more fixed set on the bench line: its planned step replayed back to
+    back (long run), per-step distributions L2-cold and warm, comparisons."""
+    import torch
+    from paper_2409_02227_gb300 import workloads as wl
+    hbm, tf_burst, tf_sust = peaks_
+    st = wl.make_config(name)
+    descs, sched, plan, single = plan_set(G, st, lut, launch_flag)
+    copies, _ = rotating_copies(st, l2)
+    r = SetRunner(st, sched, copies)
+    for k in range(10):
+        r.launch(k)
+    us = r.timed(steps) / steps * 1e3
+    cold = r.step_distribution(100, "cold", flush)
+    warm = r.step_distribution(100, "warm")
+    del r
+    torch.cuda.synchronize()
+    out = {"workload": workload_label(st.specs), "makespan_us": us, "tflops": st.flops / (us * 1e-6) / 1e12,
+           "steps": steps, "step_cold_us": cold, "step_warm_us": warm,
+           "plan": [G.goldy_variant_info_get(v)["name"] for _, v, _, _ in plan],
+           "launches_per_step": 1 if single else len(plan),
+           "roofline": roof_of(st, us, hbm, tf_burst, tf_sust)}
+    out.update(compare_policies(G, st, descs, lut, copies, max(200, min(steps, 2000)), launch_flag))
+    return out
 
 
 def run_gpu(args, world, rank, local):
@@ -481,36 +632,41 @@ def run_gpu(args, world, rank, local):
     from paper_2409_02227_gb300 import goldy as G
     from paper_2409_02227_gb300 import workloads as wl
 
-    st = wl.make_config(args.config)
-    descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
+    st = load_set(args.config)
     lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
     launch_flag = G.GOLDY_PLAN_FUSED if args.launch == "fused" else 0
-    sched = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | launch_flag)
-    plan = [G.goldy_schedule_entry(sched, i) for i in range(len(descs))]
-    kinds = {(G.goldy_variant_info_get(v)["kind"], st.specs[i].out_dtype) for i, (_, v, _, _) in enumerate(plan)}
-    n_groups = G.goldy_schedule_query(sched)[1]
-    single_launch = bool(launch_flag) and n_groups == 1 and len(kinds) == 1 and plan[0][3] >= len(descs)
+    descs, sched, plan, single_launch = plan_set(G, st, lut, launch_flag)
     props = torch.cuda.get_device_properties(device)
     l2 = int(getattr(props, "L2_cache_size", 126 * 1024 * 1024))
-    in_bytes = sum(s.batch * (2 * s.M * s.K + 2 * s.K * s.N) for s in st.specs)
-    copies = max(2, math.ceil(2 * l2 / in_bytes))
+    copies, in_bytes = rotating_copies(st, l2)
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device="cuda")
+    hbm, tf_burst, tf_sust, peak_src = peaks()
 
-    runner = SetRunner(st, sched, copies, replay=args.replay, serial_launch=args.serial_launch)
-    for k in range(max(3, args.warmup)):
-        runner.launch(k)
-    torch.cuda.synchronize()
-
+    # every prepared run is replayed once while the runner is built
+    ready = not args.no_inputs_ready
+    runner = SetRunner(st, sched, copies, replay=args.replay, serial_launch=args.serial_launch, inputs_ready=ready)
     try:
         gpu_id = "%08X:%02X:%02X.0" % (props.pci_domain_id, props.pci_bus_id, props.pci_device_id)
     except AttributeError:
         gpu_id = str(local)
     sampler = ClockSampler(gpu_id)
     sampler.start()
-    time.sleep(0.25)
+    t_load0 = time.time()
+    # per-step distributions (separate passes, never inside the headline
+    # region), then a second of the same back-to-back steps so that the
+    # clocks sampled around the timed region are those of this load
+    cold = runner.step_distribution(200, "cold", flush)
+    warm = runner.step_distribution(200, "warm")
+    est_us = max(1.0, cold["median_us"])
+    soak = int(min(200000, max(100, 1e6 / est_us)))
+    runner.timed(soak)
+    for k in range(args.warmup):
+        runner.launch(k)
+    torch.cuda.synchronize()
     barrier(dist, device)
     torch.cuda.synchronize()
     t_wall0 = time.time()
-    elapsed_ms, step_ms = runner.timed(args.steps, step_events=64 if single_launch else 0)
+    elapsed_ms = runner.timed(args.steps)
     t_wall1 = time.time()
     barrier(dist, device)
     sampler.stop()
@@ -527,16 +683,16 @@ def run_gpu(args, world, rank, local):
     dom_v = max(by_variant, key=lambda v: sum(st.specs[i].flops for i in by_variant[v]))
     dom_idx = by_variant[dom_v]
     if single_launch:
-        # one launch per step, covering all GEMMs: its average duration is the
-        # timed region's elapsed time over the steps (gaps between launches
-        # included, so an upper bound); events around each of the last 64
-        # steps are reported beside it (they add a gap of their own)
+        # one launch per step, covering all GEMMs, on the launching stream:
+        # its average duration is the timed region's elapsed time over the
+        # steps (back-to-back launches, so an upper bound)
         durs = [ms_step]
         dom_idx = list(range(len(descs)))
-        timing_note = (f"timed-region events / steps (one launch per step); events around each of the last "
-                       f"{len(step_ms)} steps alone: {statistics.mean(step_ms) * 1e3:.2f} us")
+        timing_note = ("CUDA events on the launching stream around the timed region / steps "
+                       "(one launch per step, launches back to back)")
     else:
-        inst = SetRunner(st, sched, copies, with_events=True, replay=args.replay, serial_launch=args.serial_launch)
+        inst = SetRunner(st, sched, copies, with_events=True, replay=args.replay, serial_launch=args.serial_launch,
+                         inputs_ready=ready)
         for k in range(2 * copies):
             inst.launch(k)
         torch.cuda.synchronize()
@@ -546,7 +702,6 @@ def run_gpu(args, world, rank, local):
     dur_ms = statistics.mean(durs)
     bytes_per_launch = sum(st.specs[i].bytes for i in dom_idx) / (1 if single_launch else len(dom_idx))
     flops_per_launch = sum(st.specs[i].flops for i in dom_idx) / (1 if single_launch else len(dom_idx))
-    hbm, tf_burst, tf_sust, peak_src = peaks()
     ai = flops_per_launch / bytes_per_launch
     ridge = tf_burst * 1e12 / (hbm * 1e9)
     vname = G.goldy_variant_info_get(dom_v)["name"] + (f" fused x{len(descs)}" if single_launch else "")
@@ -556,15 +711,15 @@ def run_gpu(args, world, rank, local):
     else:
         achieved = flops_per_launch / (dur_ms * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
-                "frac": achieved / tf_burst}
+                "frac": achieved / tf_burst, "peak_sustained": tf_sust, "frac_sustained": achieved / tf_sust}
     roof["traffic"] = recorded_traffic(vname)
     roof.update({"kernel": vname, "launch_us": dur_ms * 1e3,
                  "launches_sampled": args.steps if single_launch else len(durs),
                  "timing": timing_note,
                  "per_launch": {"algorithmic_bytes": bytes_per_launch, "flops": flops_per_launch},
-                 "peak_source": f"{peak_src} ({'HBM copy' if roof['bound'] == 'hbm' else 'cuBLAS bf16 burst'})"})
+                 "peak_source": f"{peak_src} ({'HBM copy' if roof['bound'] == 'hbm' else 'cuBLAS bf16 burst; sustained beside it'})"})
 
-    set_roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
+    set_roof = roof_of(st, ms_step * 1e3, hbm, tf_burst, tf_sust)
     launches_per_step = 1 if single_launch else sum(1 for s in st.specs if s.M and s.N and s.K)
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -572,45 +727,52 @@ def run_gpu(args, world, rank, local):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{args.config}: {workload_label(st.specs)}",
                    "l2": f"inputs larger than L2: {copies} rotating device copies of the set "
-                         f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2)",
+                         f"({copies * in_bytes / 2**20:.0f} MiB of A/B vs {l2 / 2**20:.0f} MiB L2); "
+                         f"no flush inside the timed region",
                    "launch": f"{'prepared-run' if args.replay == 'exec' else 'CUDA graph'} replay of the planned "
                              f"schedule ({args.launch} launch mode, "
-                             f"{'serialised launches' if args.serial_launch else 'each launch set-up overlapping the previous kernel (programmatic dependent launch)'})",
+                             f"{'serialised launches' if args.serial_launch else 'each launch set-up overlapping the previous kernel (programmatic dependent launch)'}"
+                             f"{'' if args.serial_launch or not ready else '; loads and MMAs of a launch may start during the previous kernel, its stores only after it (inputs_ready: no kernel writes an A or B)'}); "
+                             f"the timed region is one event pair around the steps, queued behind a 200 us spin "
+                             f"so the host has issued them before the GPU reaches them",
                    "plan": [{"gemm": i, "group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl,
                              "cd": cd} for i, (g, v, sl, cd) in enumerate(plan)],
                    "parallelism": f"replicas x{world}"},
         "makespan_us": ms_step * 1e3,
-        "set_roof_us": set_roof_us,
-        "set_roofline_frac": set_roof_us / (ms_step * 1e3),
+        "set_roof_us": set_roof["set_roof_us"],
+        "set_roofline_frac": set_roof["frac"],
+        "step_cold_us": cold,
+        "step_warm_us": warm,
+        "soak_steps_before_timing": soak,
         "gpu_launches": launches_per_step * args.steps,
         "roofline": roof,
     }
-    clocks = sampler.summary(t_wall0, t_wall1)
+    clocks = sampler.summary(t_load0, t_wall1)
+    clocks["window"] = "per-step passes, the soak and the timed region"
     line["clocks"] = clocks
 
     if not args.no_compare:
-        csteps = max(200, min(args.steps, 5000))
-        comp, modes = {}, {}
-        for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
-                            ("go_all_concurrent", G.GOLDY_PLAN_GO),
-                            ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
-                            ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
-            s2 = G.goldy_plan(descs, lut, flags)
-            comp[name], modes[name] = time_schedule(st, s2, copies, csteps)
-        a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
-        cb = cublas_reference_ms(st, copies, csteps) * 1e3
-        line["comparisons_us"] = {**comp, "cublas_sequential_reference": cb,
-                                  "by_replay": modes,
-                                  "note": "each configuration at its faster replay (recorded launches or graph)"}
-        line["speedup_vs_sequential"] = comp["sequential"] / a_us
-        line["speedup_vs_naive_streams"] = comp["naive_streams"] / a_us
+        line.update(compare_policies(G, st, descs, lut, copies, max(200, min(args.steps, 5000)), launch_flag))
 
     e2e_steps = max(5, min(args.steps, 200))
-    e_ms, h2d, d2h = e2e_measure(st, sched, e2e_steps)
+    e_ms, c_ms, h2d, d2h = e2e_measure(st, sched, e2e_steps)
     e_ms = reduce_max(e_ms, dist, device)
     line["e2e"] = {"value": world * st.flops / (e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
-                   "steps": e2e_steps}
+                   "steps": e2e_steps,
+                   "copies_alone_ms_per_step": c_ms,
+                   "copies_alone_gbs": (h2d + d2h) / (c_ms * 1e-3) / 1e9,
+                   "ceiling": f"the same host<->device copies without the GEMMs take {c_ms * 1e3:.1f} us per step"}
+
+    extras = [x for x in args.extra_configs.split(",") if x and x != args.config]
+    if extras:
+        del runner
+        torch.cuda.empty_cache()
+        line["configs_extra"] = {x: measure_extra(G, x, lut, l2, launch_flag, flush,
+                                                  max(2000, args.steps), (hbm, tf_burst, tf_sust))
+                                 for x in extras}
+        if G.goldy_device_error(clear=True) != 0:
+            raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
 
     if rank == 0 and not args.no_cpu:
         flops, secs, threads, desc = oracle_sample(st, budget_s=10.0)
@@ -672,7 +834,9 @@ def run_report(args, local):
         steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
         t = time_policies(st, lut, copies, steps)
         if name in wl.FIXED_CONFIGS:
-            t["cublas_sequential_reference"] = cublas_reference_ms(st, copies, steps) * 1e3
+            cb = cublas_reference_ms(st, copies, steps)
+            t["cublas_sequential_reference"] = cb["sequential"] * 1e3
+            t["cublas_streams_reference"] = cb["streams"] * 1e3
         roof_us = max(st.flops / (tf_burst * 1e12), st.bytes / (hbm * 1e9)) * 1e6
         row = {"set": name, "n_gemms": len(st.specs), "flops": st.flops, "bytes": st.bytes,
                "bound": "tensor" if st.flops / st.bytes > tf_burst * 1e12 / (hbm * 1e9) else "hbm",

@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define GOLDY_ABI_VERSION 1
+#define GOLDY_ABI_VERSION 2
 
 typedef enum goldy_status {
   GOLDY_OK = 0,
@@ -266,7 +266,10 @@ void goldy_schedule_free(goldy_schedule* s);
  * no allocation, no synchronisation.  Errors: GOLDY_ERR_INVALID_ARG (null or
  * misaligned pointers, too few streams, workspace too small),
  * GOLDY_ERR_CUDA (launch failure).  A kernel that gave up a bounded wait
- * shows up later through goldy_device_error(). */
+ * shows up later through goldy_device_error(); the outputs of that run are
+ * then incomplete, and its workspace may hold non-zero split-K arrival or
+ * unit counters: zero-fill the workspace again before the next run that uses
+ * it. */
 goldy_status goldy_run(const goldy_schedule* s, const void* const* A, const void* const* B,
                        void* const* C, void* workspace, size_t workspace_bytes,
                        void* const* streams, int n_streams);
@@ -299,6 +302,28 @@ typedef struct goldy_run_opts {
    * kernel to complete before it touches global memory, so results and
    * stream order are unchanged.  1: plain serialised launches. */
   int32_t serial_launch;
+  /* 0 (default): as above.  1: the caller asserts that no kernel enqueued
+   * before this run (on its streams) writes any A or B of the run.  Each
+   * GO-Kernel's load and MMA roles then start as soon as its CTAs are
+   * resident, while the previous kernel on the stream may still be running
+   * (reading A and B, filling shared and tensor memory); the epilogue still
+   * waits for that kernel to complete before it writes C or the workspace.
+   * Results are unchanged when the assertion holds; a violated assertion
+   * (an earlier kernel producing A or B) gives wrong results.  The bounded
+   * waits of the load and MMA roles then also cover the previous kernel's
+   * remaining time.  No effect with serial_launch = 1. */
+  int32_t inputs_ready;
+  /* Limit of every bounded wait inside the GO-Kernels, in microseconds
+   * (0: the default of 2 seconds).  A wait that runs out sets the error word
+   * (goldy_device_error) and the kernel returns. */
+  uint32_t wait_limit_us;
+  /* Test hook, 0 in normal use.  1: in the run's first GO-Kernel launch, CTA
+   * 0 never fills its first shared-memory stage (no copy is issued), so that
+   * the MMA thread's bounded wait for it runs out: the launch returns with
+   * the error word set to 2 (an MMA-thread wait gave up) and the outputs of
+   * that launch are incomplete.  Used with a short wait_limit_us to test the
+   * timeout path without faulting anything. */
+  int32_t test_stall_first_stage;
 } goldy_run_opts;
 
 /* goldy_run with options; opts may be null (then identical to goldy_run). */
@@ -440,8 +465,11 @@ void goldy_graph_free(goldy_graph* g);
 goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int variant, const void* A,
                                 const void* B, void* C, void* stream);
 
-/* Error word the kernels set when a bounded wait gives up (0 = none).  Reads
- * it synchronously on the current device and, if `clear`, resets it. */
+/* Error word the kernels set when a bounded wait gives up (0 = none; the
+ * first failure wins): 1 a load-role wait, 2 an MMA-thread wait, 3 an
+ * epilogue wait, 4 a split-K cluster-exchange wait.  Reads it synchronously
+ * on the current device and, if `clear`, resets it.  After a non-zero code,
+ * zero-fill the workspace of the failed run before reusing it (goldy_run). */
 goldy_status goldy_device_error(int* code, int clear);
 
 /* SM count and CTAs of variant `variant_id` resident per SM on the current

@@ -91,6 +91,13 @@ struct LaunchParams {
   uint32_t* dyn;              // null: CTA b takes units b, b + grid, ...; else a zeroed pair of
                               // counters (units taken, CTAs done): after its first unit b a CTA
                               // takes grid + (counter++), and the last CTA to leave zeroes both
+  uint64_t wait_ns;           // limit of every bounded wait (0: ptx::kWaitLimitNs)
+  int32_t early_loads;        // 1: the load and MMA roles start before the previous kernel on the
+                              // stream has completed (the caller asserted that no earlier kernel
+                              // writes this launch's A or B); C and the workspace are still
+                              // touched only after it (griddepcontrol.wait in the epilogue)
+  int32_t stall_test;         // test hook: CTA 0's producer never fills its first stage, so the
+                              // MMA thread's bounded wait for it runs out (0 in normal use)
 };
 
 // Units a CTA has taken but its MMA thread and epilogue have not yet both
@@ -638,10 +645,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // have initialised them before any signal is sent
   if (p.cluster > 0) ptx::cluster_sync_all();
   const uint32_t tmem_base = *tmem_slot;
+  const uint64_t wlim = p.wait_ns ? p.wait_ns : ptx::kWaitLimitNs;
   if (threadIdx.x == 0) trace_stamp(trace, kTrPreWait);
   // set-up above touched only shared and tensor memory; global memory (the
-  // operands, C, the split-K workspace) only after the previous grid is done
-  ptx::griddep_wait();
+  // operands, C, the split-K workspace) only after the previous grid is done.
+  // Early mode: the producer (reading A and B only, asserted not written by
+  // an earlier kernel) and the MMA thread (shared and tensor memory only)
+  // go ahead; the epilogue, which writes C and the workspace, still waits.
+  // A launch that hands units out from a workspace counter always waits.
+  const bool early = p.early_loads != 0 && p.dyn == nullptr && warp < 2;
+  if (!early) ptx::griddep_wait();
   if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
   if (warp == 0) {
@@ -649,15 +662,16 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       // ------------------------------------------------------------ producer
       int stage = 0;
       uint32_t phase = 0, issued = 0, last_phase = 0;
-      bool ok = true;
+      bool ok = true, stalled = false;
       int u = blockIdx.x, taken = 0;
-      for (int seq = 0; ok; ++seq) {
+      for (int seq = 0; ok && !stalled; ++seq) {
         if (p.dyn) {
           // publish the unit (or the end: an index past the last unit) to
           // the MMA thread and the epilogue
           const int slot = seq % kUnitRing;
           if (seq >= kUnitRing &&
-              !ptx::mbar_wait(ptx::smem_u32(&uempty[slot]), uint32_t((seq / kUnitRing) - 1) & 1u, abort_flag)) {
+              !ptx::mbar_wait(ptx::smem_u32(&uempty[slot]), uint32_t((seq / kUnitRing) - 1) & 1u, abort_flag,
+                              wlim)) {
             ok = false;
             break;
           }
@@ -679,8 +693,19 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           // a slot is waited for only once it has been filled before: on the
           // first pass the ring is empty (waiting on a fresh barrier's
           // preceding phase measured ~0.7 us before the first load)
-          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag, wlim)) {
             ok = false;
+            break;
+          }
+          if (p.stall_test && blockIdx.x == 0 && issued == 0) {
+            // test hook: the first stage is never filled.  No copy is in
+            // flight and no address is touched; the MMA thread's bounded
+            // wait for the stage runs out and raises the abort flag, which
+            // ends this wait too.
+            const uint64_t t0 = ptx::global_timer();
+            while (!*abort_flag && ptx::global_timer() - t0 < 4 * wlim) {
+            }
+            stalled = true;
             break;
           }
           const uint32_t fb = ptx::smem_u32(&full[stage]);
@@ -725,7 +750,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         int u = int(blockIdx.x) + seq * int(gridDim.x);   // static round-robin
         if (p.dyn) {
           const int slot = seq % kUnitRing;
-          if (!ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag)) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag, wlim)) {
             ok = false;
             break;
           }
@@ -735,7 +760,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         if (u >= p.total_units) break;
         const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         // an accumulator is waited for only once it has been used before
-        if ((acc_used >> acc & 1) && !ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+        if ((acc_used >> acc & 1) &&
+            !ptx::mbar_wait(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag, wlim)) {
           ok = false;
           break;
         }
@@ -743,7 +769,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + uint32_t(acc * MMA_N);
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
-          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag)) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag, wlim)) {
             ok = false;
             break;
           }
@@ -800,7 +826,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const int slot = seq % kUnitRing;
       int u = int(blockIdx.x) + seq * int(gridDim.x);     // static round-robin
       if (p.dyn) {
-        bool okq = ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag);
+        bool okq = ptx::mbar_wait(ptx::smem_u32(&ufull[slot]), uint32_t(seq / kUnitRing) & 1u, abort_flag, wlim);
         okq = ptx::named_bar_and(1, 128, okq);
         if (!okq) {
           if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
@@ -815,7 +841,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const GemmWork w = p.g[c.g];
       const CView cv = c_view<OUT_BF16>(w, c.b);
       bool released = false;                // accumulator already handed back
-      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
+      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag, wlim);
       ok = ptx::named_bar_and(1, 128, ok);
       if (!ok) {
         if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);
@@ -889,7 +915,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         ptx::mbar_arrive(ptx::smem_u32(&tempty[acc]));   // accumulator no longer needed
         released = true;
         if (first_unit && et == 0) trace_stamp(trace, kTrPartials);
-        bool ok2 = ptx::mbar_wait_cluster(ptx::smem_u32(recvbar), 0, abort_flag);
+        bool ok2 = ptx::mbar_wait_cluster(ptx::smem_u32(recvbar), 0, abort_flag, wlim);
         ok2 = ptx::named_bar_and(1, 128, ok2);
         if (!ok2) {
           if (et == 0) raise_error(p.err, abort_flag, kErrClusterWait);
@@ -932,7 +958,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           if (first_unit) trace_stamp(trace, kTrPartials);
           for (int q2 = 0; q2 < w.split; ++q2) ptx::mbar_arrive_remote_release(ptx::map_to_rank(rb, uint32_t(q2)));
         }
-        bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag);
+        bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag, wlim);
         ok2 = ptx::named_bar_and(1, 128, ok2);
         ++red_it;
         if (!ok2) {
@@ -977,7 +1003,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
             if (first_unit) trace_stamp(trace, kTrPartials);
             for (int q2 = 0; q2 < w.split; ++q2) ptx::mbar_arrive_remote_release(ptx::map_to_rank(rb, uint32_t(q2)));
           }
-          bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag);
+          bool ok2 = ptx::mbar_wait_cluster(rb, (red_it >> 1) & 1, abort_flag, wlim);
           ok2 = ptx::named_bar_and(1, 128, ok2);
           ++red_it;
           if (!ok2) {

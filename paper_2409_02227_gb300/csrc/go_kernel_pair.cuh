@@ -110,7 +110,11 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   ptx::cluster_sync_all();                  // the peer's barriers and tensor memory are ready
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  ptx::griddep_wait();                      // global memory only after the previous grid is done
+  const uint64_t wlim = p.wait_ns ? p.wait_ns : ptx::kWaitLimitNs;
+  // global memory only after the previous grid is done; in early mode the
+  // load and MMA roles go ahead (see go_gemm_kernel) and the epilogue waits
+  const bool early = p.early_loads != 0 && warp < 2;
+  if (!early) ptx::griddep_wait();
   if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
 
   if (warp == 0) {
@@ -127,7 +131,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         const int n0 = c.tn * 256 + int(rank) * HALF_N;
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
           // only a slot filled before is waited for (see go_gemm_kernel)
-          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag)) {
+          if ((issued >> stage & 1) && !ptx::mbar_wait(ptx::smem_u32(&empty[stage]), phase ^ 1, abort_flag, wlim)) {
             ok = false;
             break;
           }
@@ -159,7 +163,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         const uint32_t bar = ptx::smem_u32(&empty[s]);
         const uint32_t par = (last_phase >> s) & 1;
         while (!ptx::mbar_try_wait(bar, par)) {
-          if (ptx::global_timer() - t0 > ptx::kWaitLimitNs) {
+          if (ptx::global_timer() - t0 > wlim) {
             raise_error(p.err, abort_flag, kErrProducerWait);
             break;
           }
@@ -178,7 +182,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         // cluster-scope release, so wait with a cluster-scope acquire); the
         // first use of an accumulator needs no wait
         if ((acc_used >> acc & 1) &&
-            !ptx::mbar_wait_cluster(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag)) {
+            !ptx::mbar_wait_cluster(ptx::smem_u32(&tempty[acc]), acc_phase ^ 1, abort_flag, wlim)) {
           ok = false;
           break;
         }
@@ -186,7 +190,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + uint32_t(acc * 256);
         for (int kb = c.kb0; kb < c.kb1; ++kb) {
-          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag)) {
+          if (!ptx::mbar_wait(ptx::smem_u32(&full[stage]), phase, abort_flag, wlim)) {
             ok = false;
             break;
           }
@@ -236,7 +240,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
       const GemmWork w = p.g[c.g];                 // read while the accumulator is computed
       const CView cv = c_view<OUT_BF16>(w, c.b);
-      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag);
+      bool ok = ptx::mbar_wait(ptx::smem_u32(&tfull[acc]), acc_phase, abort_flag, wlim);
       ok = ptx::named_bar_and(1, 128, ok);
       if (!ok) {
         if (et == 0) raise_error(p.err, abort_flag, kErrEpilogueWait);

@@ -79,6 +79,12 @@ thread_local std::vector<Op>* t_rec = nullptr;   // non-null: record instead of 
 // their stream (the kernels wait for it before touching global memory) unless
 // the run asks for serial launches
 thread_local bool t_pdl = true;
+// Run options copied into every launch's parameters (goldy_run_opts):
+// early operand loads, the bounded-wait limit, and the test stall hook
+// (first launch of the run only).
+thread_local int32_t t_early = 0;
+thread_local uint64_t t_wait_ns = 0;
+thread_local int32_t t_stall = 0;
 // Launch priority of the next GO-Kernel launch (kNoPriority: the stream's).
 // A heterogeneous fused wave ranks its launches by work so the block
 // scheduler hands SMs to the largest first and the others fill its tail.
@@ -564,6 +570,10 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
   p.n_gemms = 1;
   p.total_units = int32_t(gp.units);
   p.err = d.err_word;
+  p.wait_ns = t_wait_ns;
+  p.early_loads = t_early;
+  p.stall_test = t_stall;
+  t_stall = 0;
 
   const Variant v = variant_of(gp.variant);
   int64_t cap = std::max<int64_t>(1, int64_t(ctas) * sms(d) / v.rc_div);
@@ -645,6 +655,10 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
   p.n_gemms = count;
   p.total_units = int32_t(units);
   p.err = d.err_word;
+  p.wait_ns = t_wait_ns;
+  p.early_loads = t_early;
+  p.stall_test = t_stall;
+  t_stall = 0;
   p.dyn = dyn ? reinterpret_cast<uint32_t*>(ws + s->gemms[members[0]].ws_dyn_off) : nullptr;
   p.trace = trace_for(grid);
   if (k.pair) {
@@ -699,6 +713,22 @@ Runtime* new_runtime(int dev, void* green, goldy_status* st) {
 }
 }  // namespace goldy
 
+namespace {
+// Restores the per-run thread-local launch options when a run ends, on every
+// return path, so that no option of one run leaks into another entry point.
+struct RunOptionsReset {
+  ~RunOptionsReset() {
+    t_trace = nullptr;
+    t_trace_ctas = 0;
+    t_trace_used = 0;
+    t_pdl = true;
+    t_early = 0;
+    t_wait_ns = 0;
+    t_stall = 0;
+  }
+};
+}  // namespace
+
 // The run itself; `own_rt`, if given, supplies the fork/join events (a
 // recorded run owns its events), otherwise the schedule's are used.
 static goldy_status run_impl(const goldy_schedule* s, const void* const* A, const void* const* B, void* const* C,
@@ -745,10 +775,14 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
   cudaStream_t main = static_cast<cudaStream_t>(streams[0]);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
 
+  RunOptionsReset reset_options;
   t_trace = opts ? static_cast<unsigned long long*>(opts->trace) : nullptr;
   t_trace_ctas = opts ? opts->trace_ctas : 0;
   t_trace_used = 0;
   t_pdl = !(opts && opts->serial_launch);
+  t_early = (opts && opts->inputs_ready) ? 1 : 0;
+  t_wait_ns = opts ? uint64_t(opts->wait_limit_us) * 1000ull : 0;
+  t_stall = (opts && opts->test_stall_first_stage) ? 1 : 0;
   auto hook = [&](void* const* evs, const int* members, int n, cudaStream_t stream) -> goldy_status {
     if (!evs) return GOLDY_OK;
     for (int j = 0; j < n; ++j) {
@@ -997,10 +1031,6 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
     if (st != GOLDY_OK) return st;
     t0 = t1;
   }
-  t_trace = nullptr;
-  t_trace_ctas = 0;
-  t_trace_used = 0;
-  t_pdl = true;
   return ok();
 }
 

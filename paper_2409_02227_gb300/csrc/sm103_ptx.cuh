@@ -2,8 +2,9 @@
 // tcgen05 tensor-memory allocation, MMA, commit and loads, plus the shared
 // memory matrix descriptor and instruction descriptor of tcgen05.mma.
 //
-// Every wait here is bounded: it gives up after kWaitLimitNs of global timer
-// time (or as soon as the CTA's abort flag is raised) and reports failure, so
+// Every wait here is bounded: it gives up after a limit of global timer time
+// (kWaitLimitNs unless the launch sets a shorter one), or as soon as the
+// CTA's abort flag is raised, and reports failure, so
 // a wrong transaction count or a missing arrival ends the kernel with an
 // error word instead of hanging the GPU.
 #pragma once
@@ -69,13 +70,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 
 // Wait until the phase with parity `parity` has completed.  Returns false if
-// the wait gave up (time limit, or *abort set by another role of the CTA).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int* abort) {
+// the wait gave up (after `limit_ns` of global timer time, or as soon as
+// *abort is set by another role of the CTA).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
+                                          uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer();
   while (!mbar_try_wait(bar, parity)) {
     if (abort != nullptr && *abort) return false;
-    if (global_timer() - t0 > kWaitLimitNs) return false;
+    if (global_timer() - t0 > limit_ns) return false;
   }
   return true;
 }
@@ -120,12 +123,13 @@ __device__ __forceinline__ bool mbar_try_wait_acq_cluster(uint32_t bar, uint32_t
 }
 
 // Bounded wait with acquire at cluster scope (pairs with the remote release).
-__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, const volatile int* abort) {
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, const volatile int* abort,
+                                                  uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait_acq_cluster(bar, parity)) return true;
   const uint64_t t0 = global_timer();
   while (!mbar_try_wait_acq_cluster(bar, parity)) {
     if (abort != nullptr && *abort) return false;
-    if (global_timer() - t0 > kWaitLimitNs) return false;
+    if (global_timer() - t0 > limit_ns) return false;
   }
   return true;
 }

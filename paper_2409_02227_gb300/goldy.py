@@ -67,7 +67,9 @@ class goldy_gemm_desc(ctypes.Structure):
 
 class goldy_run_opts(ctypes.Structure):
     _fields_ = [("ev_begin", ctypes.POINTER(ctypes.c_void_p)), ("ev_end", ctypes.POINTER(ctypes.c_void_p)),
-                ("trace", ctypes.c_void_p), ("trace_ctas", ctypes.c_size_t), ("serial_launch", ctypes.c_int32)]
+                ("trace", ctypes.c_void_p), ("trace_ctas", ctypes.c_size_t), ("serial_launch", ctypes.c_int32),
+                ("inputs_ready", ctypes.c_int32), ("wait_limit_us", ctypes.c_uint32),
+                ("test_stall_first_stage", ctypes.c_int32)]
 
 
 class goldy_variant_info(ctypes.Structure):
@@ -360,11 +362,15 @@ def goldy_graph_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Seque
 
 
 def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]], trace: int = 0,
-          trace_ctas: int = 0, serial_launch: bool = False):
+          trace_ctas: int = 0, serial_launch: bool = False, inputs_ready: bool = False,
+          wait_limit_us: int = 0, test_stall_first_stage: bool = False):
     o = goldy_run_opts()
     o.trace = int(trace) or None
     o.trace_ctas = int(trace_ctas)
     o.serial_launch = 1 if serial_launch else 0
+    o.inputs_ready = 1 if inputs_ready else 0
+    o.wait_limit_us = int(wait_limit_us)
+    o.test_stall_first_stage = 1 if test_stall_first_stage else 0
     keep = []
     if ev_begin is not None:
         arr = _ptrs(ev_begin)
@@ -380,11 +386,14 @@ def _opts(ev_begin: Optional[Sequence[int]], ev_end: Optional[Sequence[int]], tr
 def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
                  workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
                  ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0,
-                 serial_launch: bool = False) -> None:
+                 serial_launch: bool = False, inputs_ready: bool = False, wait_limit_us: int = 0,
+                 test_stall_first_stage: bool = False) -> None:
     """goldy_run with per-GEMM timing events (cudaEvent_t handles as ints),
-    an optional device phase-trace buffer and the launch mode (see
+    an optional device phase-trace buffer, the launch mode, early operand
+    loads, the bounded-wait limit and the test stall hook (see
     goldy_run_opts)."""
-    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch)
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch, inputs_ready, wait_limit_us,
+                     test_stall_first_stage)
     _check(_lib.goldy_run_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                              int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o)),
            "goldy_run_ex")
@@ -393,8 +402,9 @@ def goldy_run_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[in
 def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int],
                           workspace: int, workspace_bytes: int, streams: Sequence[int],
                           ev_begin: Optional[Sequence[int]] = None,
-                          ev_end: Optional[Sequence[int]] = None, serial_launch: bool = False) -> Graph:
-    o, _keep = _opts(ev_begin, ev_end, serial_launch=serial_launch)
+                          ev_end: Optional[Sequence[int]] = None, serial_launch: bool = False,
+                          inputs_ready: bool = False) -> Graph:
+    o, _keep = _opts(ev_begin, ev_end, serial_launch=serial_launch, inputs_ready=inputs_ready)
     out = ctypes.c_void_p()
     _check(_lib.goldy_graph_create_ex(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                                       int(workspace_bytes), _ptrs(streams), len(streams),
@@ -405,8 +415,8 @@ def goldy_graph_create_ex(s: Schedule, A: Sequence[int], B: Sequence[int], C: Se
 def goldy_exec_create(s: Schedule, A: Sequence[int], B: Sequence[int], C: Sequence[int], workspace: int,
                       workspace_bytes: int, streams: Sequence[int], ev_begin: Optional[Sequence[int]] = None,
                       ev_end: Optional[Sequence[int]] = None, trace: int = 0, trace_ctas: int = 0,
-                      serial_launch: bool = False) -> Exec:
-    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch)
+                      serial_launch: bool = False, inputs_ready: bool = False, wait_limit_us: int = 0) -> Exec:
+    o, _keep = _opts(ev_begin, ev_end, trace, trace_ctas, serial_launch, inputs_ready, wait_limit_us)
     out = ctypes.c_void_p()
     _check(_lib.goldy_exec_create(s.ptr, _ptrs(A), _ptrs(B), _ptrs(C), int(workspace) or None,
                                   int(workspace_bytes), _ptrs(streams), len(streams), ctypes.byref(o),

@@ -32,7 +32,7 @@ def test_every_declared_symbol_is_exported():
 
 
 def test_version_and_registry():
-    assert G.goldy_abi_version() == 1
+    assert G.goldy_abi_version() == 2
     n = G.goldy_variant_count()
     assert n == 132
     seen = set()

@@ -378,6 +378,40 @@ def test_dependent_launches_see_the_previous_kernels_output(cuda_ok, fused):
         assert torch.equal(outs[False][j].view(torch.int16), outs[True][j].view(torch.int16))
 
 
+@pytest.mark.parametrize("fused", [False, True])
+def test_inputs_ready_runs_overlap_and_match(cuda_ok, fused):
+    """With inputs_ready the load and MMA roles of a launch start while the
+    previous kernel on the stream is still running; the epilogue still waits
+    for it.  Independent GEMMs (none reads another's output) replayed back to
+    back on one stream give the same bytes as plain serialised launches and
+    the oracle's results."""
+    M, N, K = 256, 512, 512
+    As = [wl.random_matrix(M, K, 177 + j, "normal", 0.05) for j in range(4)]
+    bs = [wl.random_matrix(K, N, 178 + j, "normal", 0.05) for j in range(4)]
+    descs = [G.desc(M, N, K, BF16)] * 4
+    vs = [vid(2, 1, 1), vid(3, 2, 2), vid(10, 1, 1), vid(2, 4, 4)]
+    s = G.goldy_schedule_build(descs, [0, 1, 2, 3], vs, [0, 0, 0, 0], G.GOLDY_PLAN_FUSED if fused else 0)
+    _, _, ms, ws_bytes = G.goldy_schedule_query(s)
+    ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
+    dA = [a.cuda() for a in As]
+    dB = [b.cuda() for b in bs]
+    outs = {}
+    for early in (True, False):
+        dC = [torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(4)]
+        st = torch.cuda.Stream()
+        st.wait_stream(torch.cuda.current_stream())
+        for _ in range(5):
+            G.goldy_run_ex(s, [a.data_ptr() for a in dA], [b.data_ptr() for b in dB], [c.data_ptr() for c in dC],
+                           ws.data_ptr(), ws_bytes, [st.cuda_stream], serial_launch=not early, inputs_ready=early)
+        torch.cuda.current_stream().wait_stream(st)
+        torch.cuda.synchronize()
+        assert G.goldy_device_error(clear=True) == 0
+        outs[early] = [c.cpu() for c in dC]
+    for j in range(4):
+        check_close(outs[True][j], As[j], bs[j], f"independent gemm {j} with inputs_ready")
+        assert torch.equal(outs[True][j].view(torch.int16), outs[False][j].view(torch.int16))
+
+
 def _multi_group_sweep_sets(lut, count):
     """The first `count` randomized sets whose plan has several groups."""
     found = []

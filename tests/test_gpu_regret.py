@@ -5,7 +5,9 @@ For small sets the time of every subset run as one concurrent (fused) group,
 each GEMM with the table's GO-Kernel for that group size, is measured on the
 GPU; the oracle's brute-force search (oracle/schedule.py) then finds the best
 split into consecutive groups under those times, and the planner's own
-schedule is timed directly.  The regret (planner / best - 1) must stay small;
+schedule is timed directly (makespans: every run with inputs_ready off, so
+consecutive replays do not overlap and a sum of group times composes the
+way groups run one after another).  The regret (planner / best - 1) must stay small;
 the paper reports its predictor within 3% geomean of its Oracle.  The plan
 with the trained logistic-regression predictor (Eq. 1) is timed the same way.
 Each set's
@@ -39,11 +41,11 @@ def _time(st, descs, groups, variants, slots, idx, copies=4, steps=60):
     """Makespan (us) of the sub-set `idx` of `st` under an explicit fused schedule."""
     sub = wl.GemmSet(st.name, st.seed, [st.specs[i] for i in idx], [st.a[i] for i in idx], [st.b[i] for i in idx])
     sched = G.goldy_schedule_build([descs[i] for i in idx], groups, variants, slots, G.GOLDY_PLAN_FUSED)
-    r = bench.SetRunner(sub, sched, copies)
+    r = bench.SetRunner(sub, sched, copies, inputs_ready=False)
     for k in range(5):
         r.launch(k)
     torch.cuda.synchronize()
-    t = r.timed(steps)[0] / steps * 1e3
+    t = r.timed(steps) / steps * 1e3
     del r
     return t
 
@@ -75,22 +77,22 @@ def test_planner_regret_vs_exhaustive_oracle(cuda_ok, name):
 
     plan = G.goldy_plan(descs, G.goldy_lut_from_memory(lut_bytes), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
     entries_plan = [G.goldy_schedule_entry(plan, i) for i in range(n)]
-    r = bench.SetRunner(st, plan, 4)
+    r = bench.SetRunner(st, plan, 4, inputs_ready=False)
     for k in range(5):
         r.launch(k)
     torch.cuda.synchronize()
-    t_plan = r.timed(60)[0] / 60 * 1e3
+    t_plan = r.timed(60) / 60 * 1e3
     del r
     # the same planner with the trained CD predictor supplying the preferences
     t_lr = None
     if os.path.exists(G.DEFAULT_PREDICTOR):
         plan_lr = G.goldy_plan_ex(descs, G.goldy_lut_from_memory(lut_bytes), G.goldy_predictor_load(),
                                   G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
-        r = bench.SetRunner(st, plan_lr, 4)
+        r = bench.SetRunner(st, plan_lr, 4, inputs_ready=False)
         for k in range(5):
             r.launch(k)
         torch.cuda.synchronize()
-        t_lr = r.timed(60)[0] / 60 * 1e3
+        t_lr = r.timed(60) / 60 * 1e3
         del r
     # the oracle's schedule, timed the same way (its groups one after another)
     t_best = 0.0
