@@ -67,6 +67,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-inputs-ready", action="store_true",
                     help="do not let a launch's loads and MMAs start during the previous kernel's tail "
                          "(goldy_run_opts.inputs_ready = 0)")
+    ap.add_argument("--soak", type=float, default=1.0,
+                    help="seconds of the same steps run right before the timed region (sustained clocks)")
     ap.add_argument("--no-compare", action="store_true", help="skip sequential/naive/cuBLAS comparisons")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--batched-study", default=None, metavar="FILE",
@@ -206,9 +208,11 @@ def recorded_traffic(variant_name: str):
             t = json.load(f)
     except (OSError, ValueError):
         return None
-    if t.get("csrc_hash") != csrc_hash() or t.get("variant") != variant_name:
-        return None
-    return t.get("dram_bytes_per_launch")
+    h = csrc_hash()
+    for e in t.get("entries", []):
+        if e.get("csrc_hash") == h and e.get("variant") == variant_name:
+            return e.get("dram_bytes_per_launch")
+    return None
 
 
 def workload_label(specs) -> str:
@@ -430,11 +434,22 @@ def percentiles(xs):
     return {"median_us": q(0.5), "p10_us": q(0.1), "p90_us": q(0.9), "reps": len(xs)}
 
 
-def time_schedule(st, sched, copies, steps):
+def soak(runner, seconds):
+    """About `seconds` of the runner's steps back to back (untimed), so that
+    the clocks a following timed region runs at are those of this load."""
+    if seconds <= 0:
+        return
+    est_ms = max(1e-3, runner.timed(20) / 20)
+    runner.timed(int(min(200000, max(20, seconds * 1e3 / est_ms))))
+
+
+def time_schedule(st, sched, copies, steps, soak_s=0.0):
     """Makespan (us) of one schedule, replayed both ways (recorded plain
     launches and a CUDA graph); each configuration is credited with its
     faster replay, so that no baseline is slowed by a launch mode that does
-    not suit it.  Returns (best, {"exec": us, "graph": us})."""
+    not suit it.  With `soak_s`, each timed region follows that long of the
+    same steps (sustained clocks, as the bench line's own region).  Returns
+    (best, {"exec": us, "graph": us})."""
     import torch
     out = {}
     for mode in ("exec", "graph"):
@@ -442,6 +457,7 @@ def time_schedule(st, sched, copies, steps):
         for k in range(10):
             r.launch(k)
         torch.cuda.synchronize()
+        soak(r, soak_s)
         out[mode] = r.timed(steps) / steps * 1e3
         del r
     return min(out.values()), out
@@ -453,7 +469,7 @@ def cublas_reference_ms(st, copies, steps):
     ``streams`` forks one stream per GEMM from the launching stream and joins
     them back (the naive all-streams launch).  Each is one CUDA graph that
     runs the set once per rotating copy (so the inputs come from HBM),
-    replayed; ms per set."""
+    replayed after ~0.3 s of the same replays; ms per set."""
     import torch
     base_a = [a.cuda() for a in st.a]
     base_b = [b.cuda() for b in st.b]
@@ -490,6 +506,17 @@ def cublas_reference_ms(st, copies, steps):
         for _ in range(3):
             g.replay()
         torch.cuda.synchronize()
+        # ~0.3 s of the same replays first (sustained clocks, like every
+        # other configuration on the line)
+        q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        q0.record()
+        for _ in range(3):
+            g.replay()
+        q1.record()
+        torch.cuda.synchronize()
+        per_ms = max(1e-3, q0.elapsed_time(q1) / 3)
+        for _ in range(int(min(20000, 300.0 / per_ms))):
+            g.replay()
         reps = max(3, steps // copies)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
@@ -504,46 +531,66 @@ def cublas_reference_ms(st, copies, steps):
 
 
 def e2e_measure(st, sched, steps):
-    """Same metric through host buffers: each step copies A, B from pinned
-    host memory, runs the schedule, and reads C back to pinned host memory.
-    Also times the copies alone (the same bytes, same streams, no GEMMs):
-    the ceiling the end-to-end number can reach on this host link."""
+    """Same metric through host buffers and the public API: every step copies
+    its A and B from pinned host memory, runs goldy_run, and reads its C back
+    to pinned host memory.  Steps are pipelined the way a serving loop would
+    run them: two device buffer sets, input copies on one copy stream, the
+    GEMMs on the run's streams, result copies on another copy stream, ordered
+    by events, so step k's input copy overlaps step k-1's GEMMs and step
+    k-2's result copy.  Also times the copies alone (same bytes, same
+    pipeline, no GEMMs): the ceiling the end-to-end number can reach on this
+    host link."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
     _, _, ms, ws_bytes = G.goldy_schedule_query(sched)
     streams = [torch.cuda.Stream() for _ in range(max(1, ms))]
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
     ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device="cuda")
     hA = [a.pin_memory() for a in st.a]
     hB = [b.pin_memory() for b in st.b]
     cdt = [torch.bfloat16 if s.out_dtype == 0 else torch.float32 for s in st.specs]
-    hC = [torch.empty(c_shape(s), dtype=d).pin_memory() for s, d in zip(st.specs, cdt)]
-    dA = [torch.empty_like(a, device="cuda") for a in st.a]
-    dB = [torch.empty_like(b, device="cuda") for b in st.b]
-    dC = [torch.empty(c_shape(s), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)]
+    hC = [[torch.empty(c_shape(s), dtype=d).pin_memory() for s, d in zip(st.specs, cdt)] for _ in range(2)]
+    dA = [[torch.empty_like(a, device="cuda") for a in st.a] for _ in range(2)]
+    dB = [[torch.empty_like(b, device="cuda") for b in st.b] for _ in range(2)]
+    dC = [[torch.empty(c_shape(s), dtype=d, device="cuda") for s, d in zip(st.specs, cdt)] for _ in range(2)]
     main = streams[0]
-    A = [a.data_ptr() for a in dA]
-    B = [b.data_ptr() for b in dB]
-    C = [c.data_ptr() for c in dC]
     sp = [s.cuda_stream for s in streams]
+    ev = lambda: torch.cuda.Event()
+    in_done = [ev(), ev()]
+    gemm_done = [ev(), ev()]
+    out_done = [ev(), ev()]
+    for e in in_done + gemm_done + out_done:
+        e.record(main)                       # created and complete: the first waits pass
 
-    def step(gemm=True):
-        with torch.cuda.stream(main):
-            for d, h in zip(dA + dB, hA + hB):
+    def step(k, gemm=True):
+        b = k % 2
+        s_in.wait_event(gemm_done[b])        # the GEMMs of step k-2 have read this buffer set
+        with torch.cuda.stream(s_in):
+            for d, h in zip(dA[b] + dB[b], hA + hB):
                 d.copy_(h, non_blocking=True)
+        in_done[b].record(s_in)
+        main.wait_event(in_done[b])
+        main.wait_event(out_done[b])         # step k-2's results have left this buffer set
         if gemm:
-            G.goldy_run(sched, A, B, C, ws.data_ptr(), ws_bytes, sp)
-        with torch.cuda.stream(main):
-            for h, d in zip(hC, dC):
+            G.goldy_run(sched, [a.data_ptr() for a in dA[b]], [x.data_ptr() for x in dB[b]],
+                        [c.data_ptr() for c in dC[b]], ws.data_ptr(), ws_bytes, sp)
+        gemm_done[b].record(main)
+        s_out.wait_event(gemm_done[b])
+        with torch.cuda.stream(s_out):
+            for h, d in zip(hC[b], dC[b]):
                 h.copy_(d, non_blocking=True)
+        out_done[b].record(s_out)
 
     def run(gemm):
-        for _ in range(3):
-            step(gemm)
+        for k in range(4):
+            step(k, gemm)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(main)
-        for _ in range(steps):
-            step(gemm)
+        s_in.wait_stream(main)
+        for k in range(steps):
+            step(k, gemm)
+        main.wait_stream(s_out)
         e1.record(main)
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / steps
@@ -551,7 +598,7 @@ def e2e_measure(st, sched, steps):
     ms_step = run(True)
     ms_copies = run(False)
     h2d = sum(a.numel() * a.element_size() for a in hA + hB)
-    d2h = sum(c.numel() * c.element_size() for c in hC)
+    d2h = sum(c.numel() * c.element_size() for c in hC[0])
     return ms_step, ms_copies, h2d, d2h
 
 
@@ -570,20 +617,24 @@ def rotating_copies(st, l2):
     return max(2, math.ceil(2 * l2 / in_bytes)), in_bytes
 
 
-def compare_policies(G, st, descs, lut, copies, csteps, launch_flag):
+def compare_policies(G, st, descs, lut, copies, csteps, launch_flag, soak_s=0.3):
+    """Every policy timed like the bench line's own region: prepared runs (or
+    graphs) over the rotating copies, back to back after ~soak_s seconds of
+    the same steps; cuBLAS, timed the same way, as a reference point."""
     comp, modes = {}, {}
     for name, flags in (("sequential", G.GOLDY_PLAN_SEQUENTIAL), ("naive_streams", G.GOLDY_PLAN_DEFAULT),
                         ("go_all_concurrent", G.GOLDY_PLAN_GO),
                         ("goldyloc_streams", G.GOLDY_PLAN_AUTO),
                         ("goldyloc_fused", G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)):
         s2 = G.goldy_plan(descs, lut, flags)
-        comp[name], modes[name] = time_schedule(st, s2, copies, csteps)
+        comp[name], modes[name] = time_schedule(st, s2, copies, csteps, soak_s)
     a_us = comp["goldyloc_fused" if launch_flag else "goldyloc_streams"]
     cb = cublas_reference_ms(st, copies, csteps)
     out = {"comparisons_us": {**comp, "cublas_sequential_reference": cb["sequential"] * 1e3,
                               "cublas_streams_reference": cb["streams"] * 1e3, "by_replay": modes,
-                              "note": "each configuration at its faster replay (recorded launches or graph); "
-                                      "cuBLAS (torch.matmul) is a reference point only"},
+                              "note": "each configuration at its faster replay (recorded launches or graph), "
+                                      "timed after ~0.3 s of its own steps (sustained clocks, like the line's own "
+                                      "region); cuBLAS (torch.matmul, timed the same way) is a reference point only"},
            "speedup_vs_sequential": comp["sequential"] / a_us,
            "speedup_vs_naive_streams": comp["naive_streams"] / a_us}
     return out
@@ -608,11 +659,10 @@ def measure_extra(G, name, lut, l2, launch_flag, flush, steps, peaks_):
     descs, sched, plan, single = plan_set(G, st, lut, launch_flag)
     copies, _ = rotating_copies(st, l2)
     r = SetRunner(st, sched, copies)
-    for k in range(10):
-        r.launch(k)
-    us = r.timed(steps) / steps * 1e3
     cold = r.step_distribution(100, "cold", flush)
     warm = r.step_distribution(100, "warm")
+    soak(r, 0.3)
+    us = r.timed(steps) / steps * 1e3
     del r
     torch.cuda.synchronize()
     out = {"workload": workload_label(st.specs), "makespan_us": us, "tflops": st.flops / (us * 1e-6) / 1e12,
@@ -658,8 +708,8 @@ def run_gpu(args, world, rank, local):
     cold = runner.step_distribution(200, "cold", flush)
     warm = runner.step_distribution(200, "warm")
     est_us = max(1.0, cold["median_us"])
-    soak = int(min(200000, max(100, 1e6 / est_us)))
-    runner.timed(soak)
+    soak_steps = int(min(200000, max(20, args.soak * 1e6 / est_us)))
+    runner.timed(soak_steps)
     for k in range(args.warmup):
         runner.launch(k)
     torch.cuda.synchronize()
@@ -743,7 +793,7 @@ def run_gpu(args, world, rank, local):
         "set_roofline_frac": set_roof["frac"],
         "step_cold_us": cold,
         "step_warm_us": warm,
-        "soak_steps_before_timing": soak,
+        "soak_steps_before_timing": soak_steps,
         "gpu_launches": launches_per_step * args.steps,
         "roofline": roof,
     }
@@ -762,6 +812,8 @@ def run_gpu(args, world, rank, local):
                    "steps": e2e_steps,
                    "copies_alone_ms_per_step": c_ms,
                    "copies_alone_gbs": (h2d + d2h) / (c_ms * 1e-3) / 1e9,
+                   "pipeline": "two buffer sets; step k's input copy overlaps step k-1's GEMMs and step k-2's "
+                               "result copy (copy streams for each direction, event-ordered)",
                    "ceiling": f"the same host<->device copies without the GEMMs take {c_ms * 1e3:.1f} us per step"}
 
     extras = [x for x in args.extra_configs.split(",") if x and x != args.config]
