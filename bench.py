@@ -77,6 +77,9 @@ def parse_args(argv=None):
                     help="GEMM + element-wise add co-scheduling study (JSON to FILE)")
     ap.add_argument("--scaling-study", default=None, metavar="FILE",
                     help="GPU-scaling study inside SM partitions of 1/4, 1/2 and all of the GPU (JSON to FILE)")
+    ap.add_argument("--phase-trace", action="store_true",
+                    help="instead of the JSON line: per-launch phase times (device trace) of one step of the "
+                         "planned set, replayed among back-to-back steps (markdown on stdout)")
     ap.add_argument("--report", default=None, metavar="FILE",
                     help="instead of the JSON line: time every fixed set and the 64 randomized sets "
                          "under every policy and write a JSON report to FILE (markdown table on stdout)")
@@ -876,6 +879,7 @@ def run_report(args, local):
     hbm, tf_burst, _, _ = peaks()
     l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
     rows = []
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device="cuda")
     sets = [(n, wl.make_config(n)) for n in wl.FIXED_CONFIGS]
     sets += [(f"sweep_{j:02d}", None) for j in range(wl.SWEEP_SETS)]
     for name, st in sets:
@@ -885,6 +889,13 @@ def run_report(args, local):
         copies = max(2, math.ceil(2 * l2 / in_bytes))
         steps = max(50, min(2000, int(2e5 / max(1.0, st.flops / 1e9))))
         t = time_policies(st, lut, copies, steps)
+        # single steps of the GOLDYLOC plan, each with its own events: L2-cold
+        # (flushed) and warm, median and p10 / p90
+        descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
+        r = SetRunner(st, G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED), copies)
+        step_cold = r.step_distribution(60, "cold", flush)
+        step_warm = r.step_distribution(60, "warm")
+        del r
         if name in wl.FIXED_CONFIGS:
             cb = cublas_reference_ms(st, copies, steps)
             t["cublas_sequential_reference"] = cb["sequential"] * 1e3
@@ -901,11 +912,17 @@ def run_report(args, local):
                "speedup_vs_naive_streams": t["naive_streams"] / t["goldyloc"],
                "plan": [{"group": g, "variant": G.goldy_variant_info_get(v)["name"], "slot": sl, "cd": cd}
                         for g, v, sl, cd in t["plan"]],
-               "plan_lr_differs": t.get("plan_lr", t["plan"]) != t["plan"]}
+               "plan_lr_differs": t.get("plan_lr", t["plan"]) != t["plan"],
+               "goldyloc_step_cold_us": step_cold, "goldyloc_step_warm_us": step_warm}
         rows.append(row)
+        cb_s = f"{t['cublas_sequential_reference']:.2f} / {t['cublas_streams_reference']:.2f}" \
+            if "cublas_streams_reference" in t else ""
         print(f"| {name} | {len(st.specs)} | {row['bound']} | {roof_us:.2f} | {t['goldyloc']:.2f} | "
               f"{row['tflops']:.1f} | {row['roofline_frac']:.3f} | {row['speedup_vs_sequential']:.2f} | "
-              f"{row['speedup_vs_naive_streams']:.2f} | {t.get('goldyloc_lr', float('nan')):.2f} |", flush=True)
+              f"{row['speedup_vs_naive_streams']:.2f} | {t.get('goldyloc_lr', float('nan')):.2f} | "
+              f"{step_cold['median_us']:.2f} ({step_cold['p10_us']:.2f}-{step_cold['p90_us']:.2f}) | "
+              f"{step_warm['median_us']:.2f} ({step_warm['p10_us']:.2f}-{step_warm['p90_us']:.2f}) | {cb_s} |",
+              flush=True)
         del st
         torch.cuda.empty_cache()
     sweep = [r for r in rows if r["set"].startswith("sweep")]
@@ -928,6 +945,72 @@ def run_report(args, local):
     print(json.dumps(summary), flush=True)
     with open(args.report, "w") as f:
         json.dump({"rows": rows, "summary": summary, "peaks": {"hbm_gbs": hbm, "bf16_tflops": tf_burst}}, f, indent=1)
+    return 0
+
+
+TRACE_PHASES = (  # (slot, name) of goldy_run_opts.trace, in the order they happen
+    (0, "CTA start"), (10, "set-up done (before the dependency wait)"), (11, "producer starts"),
+    (2, "first stage's loads issued"), (3, "first stage landed (MMA thread)"),
+    (1, "epilogue past the dependency wait"), (4, "first accumulator committed"),
+    (5, "first accumulator seen by the epilogue"), (6, "split-K partial staged / sent"),
+    (7, "split-K partials received / arrival counted"), (8, "first unit stored"), (9, "CTA done"))
+
+
+def run_phase_trace(args, local):
+    """One step of the planned set traced on the device (%globaltimer stamps
+    per CTA, goldy_run_opts.trace) while it runs among back-to-back steps the
+    way the bench line replays them; per launch, the median and p90 over its
+    CTAs of each phase, in us from the step's first CTA start."""
+    import numpy as np
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2409_02227_gb300 import goldy as G
+    st = load_set(args.config)
+    lut = G.goldy_lut_load(args.lut or G.DEFAULT_LUT)
+    launch_flag = G.GOLDY_PLAN_FUSED if args.launch == "fused" else 0
+    descs, sched, plan, single = plan_set(G, st, lut, launch_flag)
+    l2 = int(getattr(torch.cuda.get_device_properties(local), "L2_cache_size", 126 * 2 ** 20))
+    copies, _ = rotating_copies(st, l2)
+    ready = not args.no_inputs_ready
+    r = SetRunner(st, sched, copies, serial_launch=args.serial_launch, inputs_ready=ready)
+    us = r.timed(200) / 200 * 1e3
+    cta_cap = 1 << 16
+    tr = torch.zeros(cta_cap * 16, dtype=torch.int64, device="cuda")
+    A, B, C = r.copies[0]
+    ex = G.goldy_exec_create(sched, [a.data_ptr() for a in A], [b.data_ptr() for b in B], [c.data_ptr() for c in C],
+                             r.ws.data_ptr(), r.ws_bytes, [x.cuda_stream for x in r.streams], trace=tr.data_ptr(),
+                             trace_ctas=cta_cap, serial_launch=args.serial_launch, inputs_ready=ready)
+    r.spin(200)
+    for k in range(1, 12):             # copies 1.., the traced step (copy 0) in the middle
+        r.launch(k if k % copies else k + 1)
+        if k == 6:
+            G.goldy_exec_launch(ex)
+    torch.cuda.synchronize()
+    if G.goldy_device_error(clear=True) != 0:
+        raise RuntimeError("a GO-Kernel reported a bounded-wait timeout")
+    a = tr.view(cta_cap, 16).cpu().numpy().astype(np.int64)
+    launches, off = [], 0
+    while off < cta_cap and a[off, 12] > 0:
+        g = int(a[off, 12])
+        launches.append(a[off:off + g])
+        off += g
+    t0 = min(int(l[:, 0].min()) for l in launches)
+    names = [G.goldy_variant_info_get(v)["name"] for _, v, _, _ in plan]
+    print(f"# Phase trace: {args.config} ({workload_label(st.specs)})\n")
+    print(f"Plan: {', '.join(sorted(set(names)))}; {len(launches)} launch(es) per step; "
+          f"back-to-back step time {us:.2f} us ({'inputs_ready' if ready else 'no inputs_ready'}).\n")
+    for j, l in enumerate(launches):
+        print(f"Launch {j}: grid {len(l)} CTAs, {int(l[:, 14].sum())} units, SMs used {len(set(l[:, 15].tolist()))}\n")
+        print("| phase | median us | p90 us |")
+        print("|---|---|---|")
+        for slot, name in TRACE_PHASES:
+            v = l[:, slot]
+            v = v[v > 0]
+            if v.size == 0:
+                continue
+            x = (v - t0) / 1e3
+            print(f"| {name} | {np.median(x):.2f} | {np.percentile(x, 90):.2f} |")
+        print()
     return 0
 
 
@@ -1145,6 +1228,8 @@ def main(argv=None):
         return run_reference(args, world, rank)
     if args.report:
         return run_report(args, local)
+    if args.phase_trace:
+        return run_phase_trace(args, local)
     if args.scaling_study:
         return run_scaling_study(args, local)
     if args.corun_study:

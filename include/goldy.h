@@ -284,7 +284,8 @@ typedef struct goldy_run_opts {
   void* const* ev_end;
   /* Optional device buffer of unsigned 64-bit words for a phase trace: every
    * CTA of every GO-Kernel launch writes 16 words at trace[cta * 16 + k]
-   * (k: 0 entry, 1 set-up done, 2 first TMA load, 3 first full stage seen by
+   * (k: 0 entry, 1 set-up done and the epilogue past the wait for the
+   * previous kernel, 2 first TMA load, 3 first full stage seen by
    * the MMA thread, 4 first accumulator committed, 5 first accumulator seen
    * by the epilogue, 6 split-K partial stored, 7 split-K arrival counted,
    * 8 first unit stored, 9 exit, 10 set-up done before waiting for the

@@ -109,7 +109,7 @@ constexpr int kUnitRing = 8;
 // Phase trace (optional, for profiling): %globaltimer stamps per CTA.
 enum : int {
   kTrStart = 0,        // kernel entry
-  kTrSetup = 1,        // barriers initialised, tensor memory allocated
+  kTrSetup = 1,        // the epilogue is past the wait for the previous grid (set-up done)
   kTrFirstLoad = 2,    // producer issued its first TMA load
   kTrFirstFull = 3,    // MMA thread saw its first full stage
   kTrFirstMmaDone = 4, // MMA thread committed its first accumulator
@@ -655,7 +655,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // A launch that hands units out from a workspace counter always waits.
   const bool early = p.early_loads != 0 && p.dyn == nullptr && warp < 2;
   if (!early) ptx::griddep_wait();
-  if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
+  if (threadIdx.x == 64) trace_stamp(trace, kTrSetup);   // the first epilogue thread always waits
 
   if (warp == 0) {
     if (lane == 0) {

@@ -115,7 +115,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   // load and MMA roles go ahead (see go_gemm_kernel) and the epilogue waits
   const bool early = p.early_loads != 0 && warp < 2;
   if (!early) ptx::griddep_wait();
-  if (threadIdx.x == 0) trace_stamp(trace, kTrSetup);
+  if (threadIdx.x == 64) trace_stamp(trace, kTrSetup);   // the first epilogue thread always waits
 
   if (warp == 0) {
     if (lane == 0) {

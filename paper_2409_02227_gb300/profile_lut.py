@@ -31,7 +31,13 @@ prepared runs (recorded plain launches, the way the benchmark replays a step)
 back to back on one stream, as the paper ran GEMMs back to back on each
 stream (Sec. 5.3), rotating over disjoint copies of the operands so that they
 come from HBM as in the benchmark (inputs rotated past twice the L2); the
-median of several repetitions of a timed batch.
+median of several repetitions of a timed batch.  Runs are recorded without
+inputs_ready, so that one replay does not overlap the next: a co-run's time
+is the makespan of its CD GEMMs, as the paper measures it (with overlapping
+replays, kernels whose small grids let consecutive co-runs run side by side
+win, and the table then chose worse kernels for heterogeneous waves, whose
+launches do not overlap across steps: randomized sets 0.358 -> 0.349 of
+roofline, hetero_pair 45.8 -> 52.8 us); ``--inputs-ready`` profiles with it.
 Results are appended to a JSONL log bucket by bucket, so an interrupted run
 resumes where it stopped; the LUT file is written at the end.
 
@@ -144,9 +150,10 @@ class Bench:
     operands from HBM."""
 
     def __init__(self, M: int, N: int, K: int, out: int, copies: int = 16, seed: int = 0, partition=None,
-                 rotate: bool = True, max_bytes: int = 6 << 30):
+                 rotate: bool = True, max_bytes: int = 6 << 30, inputs_ready: bool = False):
         self.M, self.N, self.K, self.out = M, N, K, out
         self.partition = partition
+        self.inputs_ready = inputs_ready
         cdt = torch.float32 if out == G.GOLDY_F32 else torch.bfloat16
         per = 2 * M * K + 2 * K * N
         cbytes = M * N * (4 if out == G.GOLDY_F32 else 2)
@@ -189,7 +196,7 @@ class Bench:
             execs.append(G.goldy_exec_create(sched, [a.data_ptr() for a in self.A[lo:hi]],
                                              [b.data_ptr() for b in self.B[lo:hi]],
                                              [c.data_ptr() for c in self.C[lo:hi]], ws.data_ptr(), ws_bytes,
-                                             self.part_streams[:max(1, ms)]))
+                                             self.part_streams[:max(1, ms)], inputs_ready=self.inputs_ready))
         est = max(G.goldy_exec_time(execs, min(groups, 3 if samples else 1), 1) * 1e3, 1.0)
         if samples == 0:
             if est >= target_us:
@@ -213,13 +220,13 @@ def pick_variant(times: Dict[int, Sequence[float]]) -> int:
     return min(times, key=lambda v: (score[v], v))
 
 
-def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) -> dict:
+def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None, inputs_ready: bool = False) -> dict:
     """Steps 1 and 2 for one bucket, at each of its sample points; a variant's
     score is its mean time relative to the fastest candidate at each point,
     so that the choice holds across the bucket, not at one shape only."""
     points = bucket_points(key)
     M, N, K, out = points[0]
-    benches = [Bench(*pt, partition=partition) for pt in points]
+    benches = [Bench(*pt, partition=partition, inputs_ready=inputs_ready) for pt in points]
     cands = sorted(set().union(*[set(candidates(pt[0], pt[1], pt[2], sm_count)) for pt in points]))
     rows = []
 
@@ -242,7 +249,8 @@ def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None) 
     speedup = {cd: sum(cd * t1 / tc for t1, tc in zip(t_cd[1], t_cd[cd])) / len(points) for cd in CD_CLASSES}
     pref = preferred_cd(speedup)
     rec = {"key": list(key), "shape": [M, N, K, out], "points": [list(pt) for pt in points], "pref_cd": pref,
-           "launch": "fused" if fused else "streams", "variants": [go[c] for c in CD_CLASSES],
+           "launch": "fused" if fused else "streams", "inputs_ready": bool(inputs_ready),
+           "variants": [go[c] for c in CD_CLASSES],
            "t_us": {str(c): t_cd[c][0] for c in CD_CLASSES},
            "t_us_points": {str(c): t_cd[c] for c in CD_CLASSES},
            "speedup": {str(c): speedup[c] for c in CD_CLASSES}, "rows": rows}
@@ -376,18 +384,19 @@ def rebuild_lut(profile_path: str, out_path: str, corun_path: str = None, sm_cou
     return len(entries)
 
 
-def profile_dataset_gemm(shape, lut, log, fused: bool = True) -> dict:
+def profile_dataset_gemm(shape, lut, log, fused: bool = True, inputs_ready: bool = False) -> dict:
     """Training record for the CD predictor (Sec. 4.3): time CD copies of one
     GEMM co-running with the table's GO-Kernel for each CD class (the kernels
     the planner would pick), CD in (1, 2, 4, 8, 16)."""
     M, N, K, out = shape
     pref, variants = G.goldy_lut_lookup(lut, G.desc(M, N, K, out))
-    bench = Bench(M, N, K, out)
+    bench = Bench(M, N, K, out, inputs_ready=inputs_ready)
     t = {}
     for c, v in zip(CD_CLASSES, variants):
         t[c] = bench.time_us(v, c, True, target_us=1000.0, fused=fused, samples=0)
     rec = {"shape": [M, N, K, out], "variants": variants, "lut_pref_cd": pref,
-           "launch": "fused" if fused else "streams", "t_us": {str(c): t[c] for c in CD_CLASSES}}
+           "launch": "fused" if fused else "streams", "inputs_ready": bool(inputs_ready),
+           "t_us": {str(c): t[c] for c in CD_CLASSES}}
     log.write(json.dumps(rec) + "\n")
     log.flush()
     del bench
@@ -395,7 +404,8 @@ def profile_dataset_gemm(shape, lut, log, fused: bool = True) -> dict:
     return rec
 
 
-def run_dataset(path: str, total: int, lut_path: str, fused: bool, time_budget: float) -> int:
+def run_dataset(path: str, total: int, lut_path: str, fused: bool, time_budget: float,
+                inputs_ready: bool = False) -> int:
     done = set()
     if os.path.exists(path):
         for line in open(path):
@@ -410,7 +420,7 @@ def run_dataset(path: str, total: int, lut_path: str, fused: bool, time_budget: 
             if time.time() - t0 > time_budget:
                 print(f"time budget reached at {i} of {len(shapes)}", flush=True)
                 return 0
-            rec = profile_dataset_gemm(sh, lut, log, fused)
+            rec = profile_dataset_gemm(sh, lut, log, fused, inputs_ready)
             if i % 50 == 0:
                 print(f"[{i + 1}/{len(shapes)}] {sh} t_us {rec['t_us']} ({time.time() - t0:.0f}s)", flush=True)
     print(f"dataset complete: {len(shapes)} GEMMs in {path}", flush=True)
@@ -462,9 +472,12 @@ def main(argv=None) -> int:
     ap.add_argument("--time-budget", type=float, default=1e9, help="stop starting buckets after this many seconds")
     ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
                     help="launch mode the co-runs of step 2 use (the mode the table will be used with)")
+    ap.add_argument("--inputs-ready", action="store_true",
+                    help="record the timed runs with inputs_ready (a replay may overlap the previous one's tail)")
     args = ap.parse_args(argv)
     if args.dataset:
-        return run_dataset(args.dataset, args.dataset_size, args.lut, args.launch == "fused", args.time_budget)
+        return run_dataset(args.dataset, args.dataset_size, args.lut, args.launch == "fused", args.time_budget,
+                           args.inputs_ready)
     if not args.out:
         ap.error("--out is required to build a table")
     if args.rebuild:
@@ -509,7 +522,8 @@ def main(argv=None) -> int:
                 print(f"time budget reached after {i} buckets", flush=True)
                 break
             tb = time.time()
-            rec = profile_bucket(key, sm_count, log, fused=args.launch == "fused", partition=partition)
+            rec = profile_bucket(key, sm_count, log, fused=args.launch == "fused", partition=partition,
+                                 inputs_ready=args.inputs_ready)
             done[key] = rec
             print(f"[{i + 1}/{len(keys)}] {key} shape {rec['shape']} pref {rec['pref_cd']} "
                   f"variants {rec['variants']} ({time.time() - tb:.1f}s)", flush=True)

@@ -304,8 +304,10 @@ def test_phase_trace_is_consistent(cuda_ok):
     assert rows.shape[0] > 0
     assert int(rows[:, 14].sum()) == 2 * 16 * 4                  # 16 tiles x split 4 per GEMM
     for r in rows.tolist():
-        assert r[0] <= r[1] <= r[2] and r[1] <= r[3] <= r[4] and r[5] <= r[8] <= r[9]
-        assert r[6] <= r[7] and r[4] <= r[5]
+        # slot 1 is stamped by the first epilogue thread, slots 2-4 by the
+        # producer and the MMA thread: ordered within each thread's sequence
+        assert r[0] <= r[1] <= r[5] and r[0] <= r[2] <= r[3] <= r[4] <= r[5] <= r[8] <= r[9]
+        assert r[6] <= r[7]
 
 
 @pytest.mark.parametrize("j", [0, 17, 63])
