@@ -577,7 +577,7 @@ goldy_status launch_gemm(DeviceState& d, const GemmPlan& gp, const void* A, cons
 
   const Variant v = variant_of(gp.variant);
   int64_t cap = std::max<int64_t>(1, int64_t(ctas) * sms(d) / v.rc_div);
-  if (scale > 0.0) cap = std::min<int64_t>(int64_t(ctas) * sms(d), int64_t(double(cap) * scale));
+  if (scale > 0.0) cap = std::min<int64_t>(int64_t(ctas) * sms(d), std::max<int64_t>(1, int64_t(double(cap) * scale)));
   if (k.pair) {
     const unsigned grid = pair_grid(gp.units, cap);
     p.trace = trace_for(grid);
@@ -621,7 +621,7 @@ goldy_status launch_fused(DeviceState& d, const goldy_schedule* s, const int* me
     if (gp.split != split) split = 0;
   }
   if (units > int64_t(1) << 30) return fail(GOLDY_ERR_UNSUPPORTED, "too many tiles in one launch");
-  if (scale > 0.0) cap = int64_t(double(cap) * scale);
+  if (scale > 0.0) cap = std::max<int64_t>(1, int64_t(double(cap) * scale));
   cap = std::min<int64_t>(cap, int64_t(ctas) * sms(d));
   const int cluster = (!k.pair && split > 1 && cluster_feasible(d, g0.kind, out_bf16, 1, split)) ? split : 0;
   const unsigned grid = k.pair ? pair_grid(units, cap) : launch_grid(units, cap, cluster);
