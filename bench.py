@@ -842,7 +842,9 @@ def run_gpu(args, world, rank, local):
 
 
 def time_policies(st, lut, copies, steps):
-    """Makespan (us) of one set under each policy, timed like the main line."""
+    """Makespan (us) of one set under each policy, timed like the main line
+    (each timed region after 0.1 s of its own steps: a GPU left idle while the
+    host builds the next set's runs starts below its clocks)."""
     import torch
     from paper_2409_02227_gb300 import goldy as G
     descs = [G.desc(s.M, s.N, s.K, s.out_dtype, batch=s.batch) for s in st.specs]
@@ -860,7 +862,7 @@ def time_policies(st, lut, copies, steps):
             sched = G.goldy_plan_ex(descs, lut, predictor, flags)
         else:
             sched = G.goldy_plan(descs, lut, flags)
-        out[name], out.setdefault("by_replay", {})[name] = time_schedule(st, sched, copies, steps)
+        out[name], out.setdefault("by_replay", {})[name] = time_schedule(st, sched, copies, steps, soak_s=0.1)
         if name in ("goldyloc", "goldyloc_lr"):
             out["plan" if name == "goldyloc" else "plan_lr"] = [G.goldy_schedule_entry(sched, i)
                                                                  for i in range(len(descs))]

@@ -81,7 +81,14 @@ typedef struct goldy_graph goldy_graph;
 /* ---- planning policies (goldy_plan flags) -------------------------------
  * The comparison configurations of Sec. 5.5 through one schedule type:
  *   AUTO        the dynamic logic: preferred CD from the table, min(CD,
- *               available), heterogeneous grouping (Sec. 4.3, Sec. 6.7)
+ *               available), heterogeneous grouping (Sec. 4.3, Sec. 6.7);
+ *               then, in each wave (a group's members taken CD at a time,
+ *               in launch order), a GEMM takes the kernel kind of the
+ *               wave's largest GEMM (no K split, that kernel's grid cap)
+ *               when the kind suits it — same C dtype, K no longer than the
+ *               largest's, M >= 128 for a CTA-pair kind, M <= 2 x the tile
+ *               rows for a transposed skinny-M kind, M >= 64 otherwise —
+ *               so that a fused wave runs as fewer launches
  *   SEQUENTIAL  isolation-tuned kernels one after another ("sequential")
  *   DEFAULT     isolation-tuned kernels, every GEMM at once on its own stream
  *               ("default", the naive all-streams launch)

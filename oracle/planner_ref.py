@@ -30,6 +30,14 @@ from the table:
 5. Inside a group GEMMs take stream slots round-robin (member j -> slot
    j mod CD), so at most CD run at once; each GEMM runs the table's kernel for
    the smallest CD class (1, 2, 4, 8, 16) not below the group's CD.
+6. One kernel kind per wave (this build's rule for its fused launches, not
+   the paper's): under the automatic policy, in each wave (a group's members
+   taken CD at a time, in launch order) every GEMM other than the wave's
+   largest (most FLOPs, ties: the first) takes the largest one's kernel kind,
+   with no K split and the same grid-cap constraint, when that kind suits it:
+   the same output dtype, K no longer than the largest one's, and M within
+   the kind's reach (CTA-pair kind: M >= 128; transposed skinny-M kind:
+   M <= 2 x its tile rows; other kinds: M >= 64).
 
 Forced policies give the paper's comparison configurations through the same
 schedule type (Sec. 5.5): ``sequential`` (isolation-tuned kernels one after
@@ -153,6 +161,56 @@ def lookup(entries: Sequence[Entry], key) -> Entry:
     return best
 
 
+# Kernel kinds of the variant registry, written out from the library's
+# documented layout (variant id = (kind * 4 + split index) * 3 + grid-cap
+# index): kind -> (tensor-core tile columns, transposed skinny-M tile, CTA
+# pair).  Transposed kinds cover mma_n rows of C per tile.
+KINDS = {
+    0: (64, False, False), 1: (64, False, False), 2: (128, False, False), 3: (128, False, False),
+    4: (256, False, False), 5: (256, False, False), 6: (32, True, False), 7: (32, True, False),
+    8: (64, True, False), 9: (64, True, False), 10: (256, False, True),
+}
+
+
+def kind_of(variant: int) -> int:
+    return variant // 12
+
+
+def same_kind_variant(kind: int, like_variant: int) -> int:
+    """Variant of `kind` with no K split and the grid-cap index of `like_variant`."""
+    return (kind * 4 + 0) * 3 + like_variant % 3
+
+
+def kind_suits(kind: int, M: int) -> bool:
+    mma_n, swap, pair = KINDS[kind]
+    if pair:
+        return M >= 128
+    if swap:
+        return M <= 2 * mma_n
+    return M >= 64
+
+
+def one_kind_per_wave(descs: Sequence["Desc"], groups):
+    """Rule 6 over groups given as (cd, members, variants); returns new groups."""
+    out = []
+    for cd, members, variants in groups:
+        var = dict(zip(members, variants))
+        for w0 in range(0, len(members), max(1, cd)):
+            wave = members[w0:w0 + max(1, cd)]
+            flops = [2 * descs[i].M * descs[i].N * descs[i].K * descs[i].batch for i in wave]
+            dom = wave[flops.index(max(flops))]            # the first of the largest
+            kd = kind_of(var[dom])
+            for i in wave:
+                if i == dom or kind_of(var[i]) == kd:
+                    continue
+                if descs[i].out_dtype != descs[dom].out_dtype or descs[i].K > descs[dom].K:
+                    continue
+                if kind_suits(kd, descs[i].M):
+                    var[i] = same_kind_variant(kd, var[dom])
+        out.append((cd, members, [var[i] for i in members]))
+    return out
+
+
 def cd_class_index(cd: int) -> int:
     for idx, c in enumerate(CD_CLASSES):
         if cd <= c:
@@ -219,6 +277,7 @@ def plan(descs: Sequence[Desc], lut_bytes: bytes, flags: int = 0):
             cd = max(1, min(cd, MAX_STREAMS))
             ci = cd_class_index(cd)
             groups.append((cd, members, [ents[i].variants[ci] for i in members]))
+        groups = one_kind_per_wave(descs, groups)
 
     per_gemm = [None] * n
     for g, (cd, members, variants) in enumerate(groups):

@@ -215,6 +215,7 @@ def _plan_with_prefs(descs, entries, prefs, flags):
         cd = max(1, min(cd, pr.MAX_STREAMS))
         ci = pr.cd_class_index(cd)
         groups.append((cd, members, [ents[i].variants[ci] for i in members]))
+    groups = pr.one_kind_per_wave(descs, groups)
     per_gemm = [None] * n
     for g, (cd, members, variants) in enumerate(groups):
         for j, (i, v) in enumerate(zip(members, variants)):

@@ -384,6 +384,47 @@ void finalize_schedule(goldy_schedule* s) {
 
 }  // namespace goldy
 
+// A wave of a group (its members taken CD at a time, in launch order) that
+// mixes kernel kinds runs one launch per kind side by side in the fused
+// launch mode, and its smaller launches mostly wait for SMs in the largest
+// one's tail.  Under the automatic policy a GEMM of a wave therefore takes
+// the kernel kind of the wave's largest GEMM (most FLOPs; ties: the first in
+// launch order) — without K split, at that kernel's grid-cap constraint —
+// when that kind suits it: the same output dtype, K no longer than the
+// largest GEMM's (no longer units than the launch's own), and M within the
+// kind's reach (a CTA-pair kind: M >= 128; a transposed skinny-M kind:
+// M <= 2 x its tile's rows; the others: M >= 64).  The wave then runs as
+// fewer, larger launches.  (This build's rule for its fused launches; the
+// paper runs one kernel per GEMM.)
+static void one_kind_per_wave(goldy_schedule* s) {
+  auto flops = [&](int i) {
+    const goldy_gemm_desc& d = s->gemms[i].desc;
+    return (unsigned __int128)2 * uint64_t(d.M) * uint64_t(d.N) * uint64_t(d.K) * uint64_t(d.batch);
+  };
+  for (const Group& grp : s->groups) {
+    const size_t size = grp.members.size();
+    const size_t cd = size_t(std::max(1, grp.cd));
+    for (size_t w0 = 0; w0 < size; w0 += cd) {
+      const size_t w1 = std::min(size, w0 + cd);
+      int dom = grp.members[w0];
+      for (size_t j = w0 + 1; j < w1; ++j)
+        if (flops(grp.members[j]) > flops(dom)) dom = grp.members[j];
+      const Variant vd = variant_of(s->gemms[dom].variant);
+      const KindInfo& kd = kKinds[vd.kind];
+      const goldy_gemm_desc& dd = s->gemms[dom].desc;
+      for (size_t j = w0; j < w1; ++j) {
+        const int i = grp.members[j];
+        const goldy_gemm_desc& di = s->gemms[i].desc;
+        if (i == dom || variant_of(s->gemms[i].variant).kind == vd.kind) continue;
+        if (di.c_dtype != dd.c_dtype || di.K > dd.K) continue;
+        const bool fits = kd.pair ? di.M >= 128 : (kd.swap_ab ? di.M <= 2 * kd.mma_n : di.M >= 64);
+        if (!fits) continue;
+        s->gemms[i].variant = variant_id(vd.kind, 0, vd.id % 3);
+      }
+    }
+  }
+}
+
 static goldy_status new_schedule(const goldy_gemm_desc* descs, int n, goldy_schedule** out) {
   if (!descs || !out) return fail(GOLDY_ERR_INVALID_ARG, "null argument");
   *out = nullptr;
@@ -516,6 +557,7 @@ extern "C" goldy_status goldy_plan_ex(const goldy_gemm_desc* descs, int n, const
       s->gemms[i].slot = int(j % size_t(groups[g].cd));
     }
   }
+  if (policy == GOLDY_PLAN_AUTO) one_kind_per_wave(s);
   finalize_schedule(s);
   *out = s;
   return ok();

@@ -62,10 +62,12 @@ def test_heterogeneous_pair_paper_rule():
     L = lut((K_SMALL, 16, V_SMALL), (K_BIG, 16, V_BIG))
     descs = [D(512, 1024, 1024)] * 8 + [D(2048, 8192, 2048)] * 8
     groups, per, ms, _ = pr.plan(descs, L)
-    # members listed block by block, the bigger-FLOP block first
+    # members listed block by block, the bigger-FLOP block first; the 16
+    # run as waves of 16, so the small GEMMs take the big ones' kernel kind
+    # (rule 6: variant 24 is kind 2, no split, grid-cap index 0)
     assert groups == [(16, list(range(8, 16)) + list(range(8)))] and ms == 16
-    assert [p[1] for p in per] == [14] * 8 + [24] * 8
-    assert per[8] == (0, 24, 0) and per[0] == (0, 14, 8)
+    assert [p[1] for p in per] == [24] * 16
+    assert per[8] == (0, 24, 0) and per[0] == (0, 24, 8)
     # one of them prefers 8 -> two homogeneous groups of 8, bigger FLOPs first
     L = lut((K_SMALL, 16, V_SMALL), (K_BIG, 8, V_BIG))
     groups, per, ms, _ = pr.plan(descs, L)
@@ -94,9 +96,54 @@ def test_greedy_merge_many_keys():
     descs = [D(32, 512, 512), D(64, 512, 512), D(128, 512, 512)]
     groups, per, ms, _ = pr.plan(descs, L)
     # FLOPs order: k3 (128 rows), k2, k1.  k3+k2 -> size 2 <= min(2, 4): merge;
-    # adding k1 -> size 3 > 2: new group.
+    # adding k1 -> size 3 > 2: new group.  In the wave [2, 1] GEMM 1 (M = 64,
+    # variant 7 = kind 0) takes GEMM 2's kind 1 (variant 12 -> 12: no split,
+    # grid-cap index 0).
     assert groups == [(2, [2, 1]), (1, [0])]
-    assert per == [(1, 1, 0), (0, 7, 1), (0, 12, 0)]
+    assert per == [(1, 1, 0), (0, 12, 1), (0, 12, 0)]
+
+
+def vid(kind, split_idx, rc_idx):
+    return (kind * 4 + split_idx) * 3 + rc_idx
+
+
+def test_one_kind_per_wave_by_hand():
+    # rule 6 on hand-built groups (cd, members, variants): descs M, N, K
+    big = D(2048, 8192, 2048)                 # the wave's largest
+    pair_v = vid(10, 0, 2)                    # CTA-pair kind, grid-cap index 2
+    cases = [
+        (D(512, 1024, 1024), vid(2, 1, 1), vid(10, 0, 2)),    # suits the pair kind: moved (no split, cap of the largest)
+        (D(96, 1024, 1024), vid(2, 1, 1), vid(2, 1, 1)),      # M < 128: a pair kind does not suit it
+        (D(512, 1024, 4096), vid(2, 1, 1), vid(2, 1, 1)),     # K longer than the largest's: kept
+        (D(512, 1024, 1024, pr.DTYPE_BF16), vid(2, 1, 1), vid(2, 1, 1)),   # other output dtype: kept
+        (D(512, 1024, 1024), vid(10, 0, 0), vid(10, 0, 0)),   # already the same kind: untouched
+    ]
+    for d, v, want in cases:
+        got = pr.one_kind_per_wave([big, d], [(2, [0, 1], [pair_v, v])])
+        assert got == [(2, [0, 1], [pair_v, want])], (d, v, got)
+    # a transposed skinny-M kind as the largest's: only M <= 2 x 32 follows it
+    t32 = vid(6, 2, 1)
+    big_skinny = D(32, 8192, 4096)
+    for M, want in ((64, vid(6, 0, 1)), (65, vid(0, 0, 0))):
+        got = pr.one_kind_per_wave([big_skinny, D(M, 256, 512)], [(2, [0, 1], [t32, vid(0, 0, 0)])])
+        assert got[0][2] == [t32, want], (M, got)
+    # waves are the members taken CD at a time: with CD 1 nothing moves
+    got = pr.one_kind_per_wave([big, D(512, 1024, 1024)], [(1, [0, 1], [pair_v, vid(2, 1, 1)])])
+    assert got == [(1, [0, 1], [pair_v, vid(2, 1, 1)])]
+    # two waves of CD 2 in launch order [0, 2, 1, 3]: each has its own
+    # largest — GEMM 0 leads [0, 2]; GEMM 3 (600 rows) leads [1, 3], so GEMM
+    # 1 (kind 4) takes kind 0 with GEMM 3's grid-cap index
+    descs = [big, D(512, 1024, 1024), D(512, 1024, 1024), D(600, 1024, 1024)]
+    got = pr.one_kind_per_wave(descs, [(2, [0, 2, 1, 3], [pair_v, vid(2, 0, 0), vid(4, 1, 0), vid(0, 0, 2)])])
+    assert got == [(2, [0, 2, 1, 3], [pair_v, vid(10, 0, 2), vid(0, 0, 2), vid(0, 0, 2)])]
+    # with GEMM 3's K halved, GEMM 1 leads the second wave and GEMM 3 follows it
+    descs[3] = D(600, 1024, 512)
+    got = pr.one_kind_per_wave(descs, [(2, [0, 2, 1, 3], [pair_v, vid(2, 0, 0), vid(4, 1, 0), vid(0, 0, 2)])])
+    assert got[0][2] == [pair_v, vid(10, 0, 2), vid(4, 1, 0), vid(4, 0, 0)]
+    # equal FLOPs: the first of them in launch order leads
+    same = [D(512, 1024, 1024), D(512, 1024, 1024)]
+    got = pr.one_kind_per_wave(same, [(2, [1, 0], [vid(2, 0, 1), vid(4, 0, 0)])])
+    assert got[0][2] == [vid(2, 0, 1), vid(2, 0, 1)]
 
 
 def test_nearest_key_and_ties():
