@@ -343,6 +343,46 @@ def test_sweep_sets_through_the_predictor_plan(cuda_ok, j):
         check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} (predictor plan) gemm {i} {s.M}x{s.N}x{s.K}")
 
 
+@pytest.mark.parametrize("j", [12, 14, 17])
+def test_one_kind_per_wave_plans_match_oracle(cuda_ok, j):
+    # randomized sets in which the planner moves GEMMs of a wave to the kind
+    # of the wave's largest GEMM (set 12: two into the CTA-pair kernel, 14:
+    # seven between single-CTA kinds, 17: four into the pair kernel): every
+    # GEMM on sampled rows (first and last included) against the oracle, the
+    # plan bit-identical fused, in streams mode and as a prepared run
+    st = wl.make_sweep_set(j)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    lut = G.goldy_lut_load(G.DEFAULT_LUT)
+    fused = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    classes = (1, 2, 4, 8, 16)
+    moved = 0
+    for i, d in enumerate(descs):
+        _, v, _, cd = G.goldy_schedule_entry(fused, i)
+        table_v = G.goldy_lut_lookup(lut, d)[1][next(k for k, c in enumerate(classes) if c >= cd)]
+        moved += int(v != table_v)
+    assert moved >= 2
+    outs = [s.out_dtype for s in st.specs]
+    Lf = Launch(fused, st.a, st.b, outs)
+    Lf.run()
+    got = Lf.results()
+    rng = np.random.default_rng(4000 + j)
+    for i, s in enumerate(st.specs):
+        rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(8, s.M))]))
+        check_rows(got[i], st.a[i], st.b[i], rows, f"sweep {j} gemm {i} {s.M}x{s.N}x{s.K}")
+    streams = G.goldy_plan(descs, lut, G.GOLDY_PLAN_AUTO)
+    Ls = Launch(streams, st.a, st.b, outs)
+    Ls.run()
+    for x, y in zip(got, Ls.results()):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8))
+    for c in Lf.dC:
+        c.fill_(float("nan"))
+    x = Lf.exec()
+    G.goldy_exec_launch(x)
+    for a, b in zip(got, Lf.results()):
+        assert torch.equal(a.view(torch.uint8), b.view(torch.uint8))
+    del x
+
+
 @pytest.mark.parametrize("fused", [False, True])
 def test_dependent_launches_see_the_previous_kernels_output(cuda_ok, fused):
     """Kernels of one stream overlap their set-up with the previous kernel
