@@ -383,6 +383,36 @@ def test_one_kind_per_wave_plans_match_oracle(cuda_ok, j):
     del x
 
 
+@pytest.mark.parametrize("j", [30, 48, 16])
+def test_few_launch_runs_on_one_stream_match(cuda_ok, j):
+    # randomized sets whose fused plan has 2 to 5 launches: with inputs_ready
+    # they go out on streams[0] alone (each wave's largest first); replayed
+    # back to back as prepared runs they give the same bytes as the forked
+    # multi-stream run without the option, and the oracle's values
+    st = wl.make_sweep_set(j)
+    descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
+    sched = G.goldy_plan(descs, G.goldy_lut_load(G.DEFAULT_LUT), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)
+    outs = [s.out_dtype for s in st.specs]
+    L = Launch(sched, st.a, st.b, outs)
+    L.run()
+    ref = L.results()
+    rng = np.random.default_rng(5000 + j)
+    for i, s in enumerate(st.specs):
+        rows = np.unique(np.concatenate([[0, s.M - 1], rng.integers(0, s.M, size=min(6, s.M))]))
+        check_rows(ref[i], st.a[i], st.b[i], rows, f"sweep {j} gemm {i}")
+    for c in L.dC:
+        c.fill_(float("nan"))
+    A, B, C = L.ptrs()
+    x = G.goldy_exec_create(sched, A, B, C, L.ws.data_ptr(), L.ws_bytes, [s.cuda_stream for s in L.streams],
+                            inputs_ready=True)
+    for _ in range(4):
+        G.goldy_exec_launch(x)
+    got = L.results()
+    for a, b in zip(got, ref):
+        assert torch.equal(a.view(torch.uint8), b.view(torch.uint8))
+    del x
+
+
 @pytest.mark.parametrize("fused", [False, True])
 def test_dependent_launches_see_the_previous_kernels_output(cuda_ok, fused):
     """Kernels of one stream overlap their set-up with the previous kernel
