@@ -134,8 +134,10 @@ const char* goldy_last_error(void);
  * A variant is one GO-Kernel configuration (Sec. 4.2): a tile shape and
  * shared-memory/tensor-memory footprint (kind), a split of the K loop, and a
  * resource constraint (RC) capping the persistent grid at the whole GPU, half
- * or a quarter of it (Sec. 4.2.1's GPU, GPU/2, GPU/4).  Kinds whose tiles are
- * computed by a CTA pair ignore the split factor (they never split K). */
+ * or a quarter of it (Sec. 4.2.1's GPU, GPU/2, GPU/4).  With a split S > 1
+ * the S K-ranges of a tile are summed in split order 0 .. S-1 (in a cluster
+ * of S CTAs, or by the last split to arrive, through the workspace; a CTA-pair
+ * kind always through the workspace). */
 typedef struct goldy_variant_info {
   int32_t id;
   int32_t kind;           /* tile/footprint family, 0 .. n_kinds-1 */

@@ -119,8 +119,6 @@ def kernel_features(M: int, N: int, variant: int, sm_count: int, batch: int = 1)
     split = SPLITS[(variant // 3) % 4]
     rc_div = RC_DIVS[variant % 3]
     rows, cols, per_sm, per_tile = KIND_GEOMETRY[kind]
-    if per_tile > 1:
-        split = 1
     tiles = batch * (-(-M // rows)) * (-(-N // cols))
     ctas = tiles * split * per_tile
     cap = max(per_tile, per_sm * sm_count // rc_div)

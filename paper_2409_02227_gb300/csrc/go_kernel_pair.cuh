@@ -14,8 +14,11 @@
 // loads complete on the even CTA's barrier), warp 1 allocates tensor memory
 // jointly with the peer and, in the even CTA, issues the MMAs and commits
 // (multicast to both CTAs' barriers), warps 2-5 drain the CTA's own half of
-// the accumulator.  Units (256 x 256 tiles) go to pairs round-robin; both CTAs
-// of a pair walk the same sequence.  Every wait is bounded; before leaving,
+// the accumulator.  Units (256 x 256 tiles, or with a K split S, S K-ranges
+// of a tile) go to pairs round-robin; both CTAs of a pair walk the same
+// sequence.  With S > 1 each CTA publishes its 128 x 256 fp32 partial to the
+// workspace and the last split to arrive for a tile half sums the S partials
+// in split order and stores C.  Every wait is bounded; before leaving,
 // each CTA waits (bounded) until every arrival the peer owes its barriers has
 // landed, then the pair meets at a cluster barrier.
 #pragma once
@@ -49,6 +52,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   uint64_t* drain = bars + 2 * STAGES + 2 * ACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);   // split-K: last arriver
   UnitTable* utab = reinterpret_cast<UnitTable*>(tmem_slot + 4);   // see go_gemm_kernel
   static_assert((2 * STAGES + 2 * ACC + 1) * 8 + 16 + MAXG * int(sizeof(UnitTable)) <= 1024, "barrier area");
   const int n_gemms = p.n_gemms;
@@ -87,6 +91,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     }
     ptx::mbar_init(ptx::smem_u32(drain), 1);
     *abort_flag = 0;
+    *last_flag = 0;
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
   }
@@ -252,7 +257,69 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       const int m0 = c.tm * 256 + int(rank) * 128;
       const int n0 = c.tn * 256;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
-      if (w.c_tma) {
+      if (w.split > 1) {
+        // ---- split-K: this CTA publishes its fp32 partial (its 128 rows of
+        // the 256 x 256 tile, layout [chunk][float4][row]) to the workspace
+        // and counts itself in; the last of the S splits to arrive for this
+        // tile half sums the S partials in split order 0, 1, ..., S-1 (its
+        // own from tensor memory) and stores C, then zeroes the counter.  No
+        // CTA waits for another.
+        constexpr int TILE_F4 = 128 * 256 / 4;
+        float4* part_base = reinterpret_cast<float4*>(w.ws_part);
+        const size_t half = size_t(c.tile) * 2 + rank;
+        float4* mine = part_base + (half * size_t(w.split) + size_t(c.s)) * TILE_F4;
+#pragma unroll 1
+        for (int c0 = 0; c0 < 256; c0 += 32) {
+          uint32_t raw[32];
+          __syncwarp();
+          ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int j4 = 0; j4 < 8; ++j4)
+            mine[((c0 / 4) + j4) * 128 + r] =
+                make_float4(__uint_as_float(raw[4 * j4]), __uint_as_float(raw[4 * j4 + 1]),
+                            __uint_as_float(raw[4 * j4 + 2]), __uint_as_float(raw[4 * j4 + 3]));
+        }
+        __threadfence();
+        ptx::named_bar_sync(1, 128);
+        if (et == 0) {
+          const uint32_t old = atomicAdd(&w.ws_cnt[half], 1u);
+          *last_flag = (old == uint32_t(w.split - 1)) ? 1 : 0;
+        }
+        ptx::named_bar_sync(1, 128);
+        if (*last_flag) {
+          __threadfence();
+          const float4* parts = part_base + half * size_t(w.split) * TILE_F4;
+#pragma unroll 1
+          for (int c0 = 0; c0 < 256; c0 += 32) {
+            uint32_t raw[32];
+            __syncwarp();
+            ptx::tmem_ld_32x32b_x32(taddr + c0, raw);
+            ptx::tmem_ld_wait();
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+#pragma unroll 1
+            for (int s2 = 0; s2 < w.split; ++s2) {
+              float4 t[8];
+#pragma unroll
+              for (int j4 = 0; j4 < 8; ++j4)
+                t[j4] = (s2 == c.s) ? make_float4(__uint_as_float(raw[4 * j4]), __uint_as_float(raw[4 * j4 + 1]),
+                                                   __uint_as_float(raw[4 * j4 + 2]), __uint_as_float(raw[4 * j4 + 3]))
+                                    : __ldcg(&parts[size_t(s2) * TILE_F4 + ((c0 / 4) + j4) * 128 + r]);
+#pragma unroll
+              for (int j4 = 0; j4 < 8; ++j4) {
+                v[4 * j4] += t[j4].x;
+                v[4 * j4 + 1] += t[j4].y;
+                v[4 * j4 + 2] += t[j4].z;
+                v[4 * j4 + 3] += t[j4].w;
+              }
+            }
+            store_chunk<false, OUT_BF16>(cv, m0, n0, r, c0, v);
+          }
+          if (et == 0) w.ws_cnt[half] = 0u;     // leave the counter zeroed for the next run
+        }
+      } else if (w.c_tma) {
         store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
       } else {
 #pragma unroll 1

@@ -53,7 +53,7 @@ inline constexpr KindInfo kKinds[kNumKinds] = {
     {"t32_half", 32, 1, 4, 2, 2, 0},
     {"t64_full", 64, 1, 8, 2, 1, 0},
     {"t64_half", 64, 1, 4, 2, 2, 0},
-    {"p256_pair", 256, 0, 6, 2, 1, 1},   // 256 x 256 tiles over a CTA pair; split-K is not used
+    {"p256_pair", 256, 0, 6, 2, 1, 1},   // 256 x 256 tiles over a CTA pair; split-K through the workspace
 };
 
 constexpr int stage_bytes(const KindInfo& k) {

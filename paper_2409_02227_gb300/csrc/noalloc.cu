@@ -97,14 +97,16 @@ extern "C" goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int vari
   gp.tiles_m = ceil_div(desc->M, tile_rows(k));
   gp.tiles_n = ceil_div(desc->N, tile_cols(k));
   gp.k_blocks = ceil_div(desc->K, kBlockK);
-  gp.split = k.pair ? 1 : int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
+  gp.split = int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
   const int64_t tiles = gp.tiles_m * gp.tiles_n;
   gp.units = desc->K > 0 ? tiles * gp.split : 0;
-  size_t need = 0, cnt_off = 0;
+  size_t need = 0, cnt_off = 0, counters = 0;
   if (gp.split > 1 && tiles > 0) {
-    const size_t part = size_t(gp.units) * kMmaM * k.mma_n * sizeof(float);
+    const size_t halves = k.pair ? 2 : 1;     // a CTA pair keeps a partial and a counter per CTA
+    const size_t part = size_t(gp.units) * halves * kMmaM * k.mma_n * sizeof(float);
     cnt_off = (part + 255) & ~size_t(255);
-    need = cnt_off + size_t(tiles) * sizeof(uint32_t);
+    counters = size_t(tiles) * halves;
+    need = cnt_off + counters * sizeof(uint32_t);
   }
   if (need > kNoAllocScratchBytes)
     return fail(GOLDY_ERR_INVALID_ARG, "this GEMM and variant need " + std::to_string(need) +
@@ -125,7 +127,7 @@ extern "C" goldy_status goldy_gemm_noalloc(const goldy_gemm_desc* desc, int vari
     gp.ws_part_off = 0;
     gp.ws_cnt_off = cnt_off;
     gp.ws_bytes = need;
-    clear_bytes = size_t(tiles) * sizeof(uint32_t);
+    clear_bytes = counters * sizeof(uint32_t);
   }
   st = launch_planned_gemm(gp, A, B, C, scratch, stream, cnt_off, clear_bytes);
   if (st != GOLDY_OK) return st;

@@ -287,7 +287,7 @@ static void lr_features(const goldy_gemm_desc& d, const LutEntry& e, int64_t sm_
     const Variant v = variant_of(e.variant[c]);
     const KindInfo& k = kKinds[v.kind];
     const int64_t per_tile = k.pair ? 2 : 1;
-    const int64_t split = k.pair ? 1 : v.split;
+    const int64_t split = v.split;
     const int64_t ctas = d.batch * ceil_div(d.M, tile_rows(k)) * ceil_div(d.N, tile_cols(k)) * split * per_tile;
     const int64_t cap = std::max<int64_t>(per_tile, int64_t(k.ctas_per_sm) * sm_count / v.rc_div);
     x[3 + 3 * c] = double(ctas);
@@ -359,15 +359,18 @@ void finalize_schedule(goldy_schedule* s) {
     gp.tiles_m = ceil_div(gp.desc.M, tile_rows(k));
     gp.tiles_n = ceil_div(gp.desc.N, tile_cols(k));
     gp.k_blocks = ceil_div(gp.desc.K, kBlockK);
-    gp.split = k.pair ? 1 : int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
+    gp.split = int(std::max<int64_t>(1, std::min<int64_t>(v.split, gp.k_blocks)));
     const int64_t tiles = gp.tiles_m * gp.tiles_n * gp.desc.batch;   // over all batch entries
     gp.units = (gp.desc.K > 0) ? tiles * gp.split : 0;
     gp.ws_part_off = gp.ws_cnt_off = gp.ws_bytes = 0;
     if (gp.split > 1 && tiles > 0) {
+      // a partial tile per unit (a CTA pair: one per CTA, 128 rows each) and
+      // an arrival counter per tile (per tile half for a pair)
+      const size_t halves = k.pair ? 2 : 1;
       gp.ws_part_off = off;
-      off = align(off + size_t(gp.units) * kMmaM * k.mma_n * sizeof(float));
+      off = align(off + size_t(gp.units) * halves * kMmaM * k.mma_n * sizeof(float));
       gp.ws_cnt_off = off;
-      off = align(off + size_t(tiles) * sizeof(uint32_t));
+      off = align(off + size_t(tiles) * halves * sizeof(uint32_t));
       gp.ws_bytes = off - gp.ws_part_off;
     }
   }
@@ -675,7 +678,7 @@ extern "C" goldy_status goldy_variant_info_get(int id, goldy_variant_info* out) 
   out->acc_stages = k.acc_stages;
   out->tmem_cols = tmem_cols(k);
   out->smem_bytes = smem_bytes(k);
-  out->split_k = k.pair ? 1 : v.split;
+  out->split_k = v.split;
   out->rc_div = v.rc_div;
   out->ctas_per_sm = k.ctas_per_sm;
   out->cta_pair = k.pair ? 2 : 1;

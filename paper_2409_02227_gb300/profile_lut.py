@@ -135,7 +135,7 @@ def candidates(M: int, N: int, K: int, sm_count: int) -> List[Tuple[int, int]]:
         cols = 128 if info["swap_ab"] else info["mma_n"]
         tiles = math.ceil(M / rows) * math.ceil(N / cols)
         for s in SPLITS:
-            if s > 1 and (info["cta_pair"] == 2 or s > k_blocks or tiles * s > 4 * sm_count):
+            if s > 1 and (s > k_blocks or tiles * s > 4 * sm_count):
                 continue
             out.append((kind, s))
     return out

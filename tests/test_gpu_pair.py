@@ -1,7 +1,7 @@
 """GPU parity of the CTA-pair GO-Kernel (256 x 256 tiles, one tcgen05 MMA
 across two SMs): ragged shapes against the fp64 oracle, exact integer
-results, several GEMMs in one fused launch, and bit-identical results alone
-vs co-scheduled."""
+results, K splits reduced through the workspace, several GEMMs in one fused
+launch, and bit-identical results alone vs co-scheduled."""
 import numpy as np
 import pytest
 import torch
@@ -46,12 +46,58 @@ def test_pair_integer_exact(cuda_ok):
     assert torch.equal(c, exact)
 
 
-def test_pair_grid_cap_and_split_ids_are_bit_exact(cuda_ok):
+def test_pair_grid_cap_is_bit_exact(cuda_ok):
     a, b = inputs(1024, 1024, 512, seed=40)
-    outs = [run_explicit([a], [b], [F32], [vid(s, rc)])[0] for s, rc in ((1, 1), (1, 2), (1, 4), (8, 1))]
+    outs = [run_explicit([a], [b], [F32], [vid(1, rc)])[0] for rc in (1, 2, 4)]
     check_close(outs[0], a, b, "pair rc1")
     for o in outs[1:]:
         assert torch.equal(outs[0], o)
+
+
+@pytest.mark.parametrize("out", [F32, BF16])
+@pytest.mark.parametrize("split", [2, 4, 8])
+@pytest.mark.parametrize("M,N,K", [(300, 320, 1472), (1024, 768, 2048), (130, 520, 448)])
+def test_pair_split_k(cuda_ok, M, N, K, split, out):
+    # split-K for the pair kind: every CTA publishes its partial, the last
+    # split to arrive sums them in split order; ragged tails, splits clamped
+    # to the K blocks (448 = 7 blocks), grid caps bit-exact, the workspace's
+    # counters back at zero after each run (a second run gives the same bytes)
+    a, b = inputs(M, N, K, seed=M + 3 * N + K + split, dist="normal", scale=0.5)
+    d = G.desc(M, N, K, out)
+    runs = []
+    for rc in (1, 4):
+        s = G.goldy_schedule_build([d], [0], [vid(split, rc)], [0])
+        L = Launch(s, [a], [b], [out])
+        for _ in range(2):
+            L.run()
+            runs.append(L.results()[0])
+    check_close(runs[0], a, b, f"pair split {split} {M}x{N}x{K}")
+    for r in runs[1:]:
+        x, y = (r, runs[0]) if r.dtype != torch.bfloat16 else (r.view(torch.int16), runs[0].view(torch.int16))
+        assert torch.equal(x, y)
+
+
+def test_pair_split_k_integer_exact_and_fused_with_others(cuda_ok):
+    # small integers are exact whatever the split; a fused launch of the pair
+    # kind with GEMMs of different splits (workspace partials of each) gives
+    # the bytes each gives alone
+    a = wl.integer_matrix(384, 2048, seed=33)
+    b = wl.integer_matrix(2048, 512, seed=34)
+    (c,) = run_explicit([a], [b], [F32], [vid(4, 1)])
+    assert torch.equal(c, (a.to(torch.int64) @ b.to(torch.int64)).to(torch.float32))
+    shapes = [(512, 1024, 2048), (300, 512, 1024), (256, 256, 512)]
+    A, B = zip(*[inputs(M, N, K, seed=60 + i, dist="normal", scale=0.1) for i, (M, N, K) in enumerate(shapes)])
+    vs = [vid(2, 1), vid(4, 1), vid(1, 1)]
+    alone = [run_explicit([A[i]], [B[i]], [F32], [vs[i]])[0] for i in range(3)]
+    descs = [G.desc(M, N, K, F32) for (M, N, K) in shapes]
+    s = G.goldy_schedule_build(descs, [0, 0, 0], vs, [0, 1, 2], G.GOLDY_PLAN_FUSED)
+    L = Launch(s, list(A), list(B), [F32] * 3)
+    for _ in range(2):
+        L.run()
+        got = L.results()
+        for i in range(3):
+            check_close(got[i], A[i], B[i], f"fused pair {i}")
+            assert torch.equal(got[i], alone[i])
 
 
 def test_pair_fused_and_co_scheduled(cuda_ok):

@@ -61,8 +61,8 @@ def test_kernel_features_hand_worked():
     # n64_full split 8, quarter GPU on 4096 x 8192: 32 x 128 tiles x 8 = 32768;
     # cap 38: 38 x 862 = 32756 < 32768 -> 863 waves
     assert P.kernel_features(4096, 8192, vid(0, 3, 2), 152) == (32768, 1, 863)
-    # the pair kind ignores a split index
-    assert P.kernel_features(300, 300, vid(10, 3, 0), 152) == (8, 1, 1)
+    # the pair kind with split 8 on 300 x 300: 2 x 2 tiles x 8 splits x 2 CTAs = 64
+    assert P.kernel_features(300, 300, vid(10, 3, 0), 152) == (64, 1, 1)
 
 
 def test_feature_vector_order():
