@@ -211,16 +211,23 @@ class Bench:
         return times[len(times) // 2]
 
 
-def pick_variant(times: Dict[int, Sequence[float]]) -> int:
-    """The variant with the smallest mean, over the sample points, of its time
-    relative to the fastest variant at that point (ties: the smaller id)."""
+def rank_variants(times: Dict[int, Sequence[float]]) -> List[int]:
+    """Variants from best to worst by the mean, over the sample points, of
+    their time relative to the fastest variant at that point (ties: the
+    smaller id)."""
     n = len(next(iter(times.values())))
     fastest = [min(ts[pi] for ts in times.values()) for pi in range(n)]
     score = {v: sum(t / f for t, f in zip(ts, fastest)) / n for v, ts in times.items()}
-    return min(times, key=lambda v: (score[v], v))
+    return sorted(times, key=lambda v: (score[v], v))
 
 
-def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None, inputs_ready: bool = False) -> dict:
+def pick_variant(times: Dict[int, Sequence[float]]) -> int:
+    """The best variant of rank_variants."""
+    return rank_variants(times)[0]
+
+
+def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None, inputs_ready: bool = False,
+                   top: int = 1) -> dict:
     """Steps 1 and 2 for one bucket, at each of its sample points; a variant's
     score is its mean time relative to the fastest candidate at each point,
     so that the choice holds across the bucket, not at one shape only."""
@@ -230,21 +237,24 @@ def profile_bucket(key, sm_count: int, log, fused: bool = True, partition=None, 
     cands = sorted(set().union(*[set(candidates(pt[0], pt[1], pt[2], sm_count)) for pt in points]))
     rows = []
 
-    def best_of(variants, copies, step, extra):
+    def ranked(variants, copies, step, extra):
         times = {v: [b.time_us(v, copies, True, fused=fused) for b in benches] for v in variants}
         for v, ts in times.items():
             for pi, t in enumerate(ts):
                 rows.append(dict(step=step, variant=v, point=pi, us=t, **extra))
-        v = pick_variant(times)
-        return v, times[v]
+        order = rank_variants(times)
+        return order, times
 
     winners = {}
     for rc in RC_DIVS:                                  # step 1
-        winners[rc] = best_of([G.variant_id(kind, split, rc) for kind, split in cands], 1, 1, {"rc": rc})
-    go = {1: winners[1][0]}
-    t_cd = {1: winners[1][1]}
+        winners[rc] = ranked([G.variant_id(kind, split, rc) for kind, split in cands], 1, 1, {"rc": rc})
+    go = {1: winners[1][0][0]}
+    t_cd = {1: winners[1][1][go[1]]}
+    # step 2 co-runs the best `top` kernels of each constraint (the paper: the best one)
+    step2 = sorted({v for rc in RC_DIVS for v in winners[rc][0][:top]})
     for cd in (2, 4, 8, 16):                            # step 2
-        go[cd], t_cd[cd] = best_of(sorted({winners[rc][0] for rc in RC_DIVS}), cd, 2, {"cd": cd})
+        order, times = ranked(step2, cd, 2, {"cd": cd})
+        go[cd], t_cd[cd] = order[0], times[order[0]]
     # speedup over running the copies one after another, averaged over the points
     speedup = {cd: sum(cd * t1 / tc for t1, tc in zip(t_cd[1], t_cd[cd])) / len(points) for cd in CD_CLASSES}
     pref = preferred_cd(speedup)
@@ -472,6 +482,9 @@ def main(argv=None) -> int:
     ap.add_argument("--time-budget", type=float, default=1e9, help="stop starting buckets after this many seconds")
     ap.add_argument("--launch", choices=["fused", "streams"], default="fused",
                     help="launch mode the co-runs of step 2 use (the mode the table will be used with)")
+    ap.add_argument("--top", type=int, default=1,
+                    help="step 2 co-runs the best TOP kernels of each resource constraint (default 1: the paper's "
+                         "single winner per constraint)")
     ap.add_argument("--inputs-ready", action="store_true",
                     help="record the timed runs with inputs_ready (a replay may overlap the previous one's tail)")
     args = ap.parse_args(argv)
@@ -523,7 +536,7 @@ def main(argv=None) -> int:
                 break
             tb = time.time()
             rec = profile_bucket(key, sm_count, log, fused=args.launch == "fused", partition=partition,
-                                 inputs_ready=args.inputs_ready)
+                                 inputs_ready=args.inputs_ready, top=args.top)
             done[key] = rec
             print(f"[{i + 1}/{len(keys)}] {key} shape {rec['shape']} pref {rec['pref_cd']} "
                   f"variants {rec['variants']} ({time.time() - tb:.1f}s)", flush=True)

@@ -71,7 +71,11 @@ def test_bucket_shapes_and_candidates():
     assert all(s in (1, 2, 4, 8) for _, s in c)
     big = {k for k, _ in P.candidates(512, 1024, 1024, 152)}
     assert not {6, 7, 8, 9} & big and 10 in big
-    assert all(s == 1 for k, s in P.candidates(512, 1024, 1024, 152) if k == 10)
+    # the pair kind splits K too: 2 x 4 tiles of 256 x 256, K = 1024 -> 16 blocks
+    assert sorted(s for k, s in P.candidates(512, 1024, 1024, 152) if k == 10) == [1, 2, 4, 8]
+    # ...but not beyond the K blocks (K = 128: 2 blocks) or 4 x the SMs of units
+    assert sorted(s for k, s in P.candidates(512, 1024, 128, 152) if k == 10) == [1, 2]
+    assert sorted(s for k, s in P.candidates(4096, 8192, 4096, 152) if k == 10) == [1]
 
 
 def _free_port():
@@ -142,3 +146,11 @@ def test_pick_variant_scores_relative_times():
     assert P.pick_variant({1: [1.0, 120.0], 2: [1.3, 100.0]}) == 1
     # ties -> smaller id
     assert P.pick_variant({9: [2.0, 4.0], 4: [2.0, 4.0]}) == 4
+
+
+def test_rank_variants_orders_by_relative_time():
+    # mean ratio to the fastest at each point: 7 (1.0, 1.4) -> 1.2; 3 (1.05, 1.0)
+    # -> 1.025; 5 (1.1, 1.2) -> 1.15; ties to the smaller id
+    times = {3: [10.5, 20.0], 7: [10.0, 28.0], 5: [11.0, 24.0], 2: [11.0, 24.0]}
+    assert P.rank_variants(times) == [3, 2, 5, 7]
+    assert P.pick_variant(times) == P.rank_variants(times)[0]
