@@ -579,7 +579,7 @@ def test_phase_trace_regions_per_launch(cuda_ok):
         rows_ = info["mma_n"] if info["swap_ab"] else (256 if info["cta_pair"] == 2 else 128)
         cols = 128 if info["swap_ab"] else info["mma_n"]
         tiles = -(-s.M // rows_) * -(-s.N // cols)
-        split = 1 if info["cta_pair"] == 2 else min(info["split_k"], -(-s.K // 64))
+        split = min(info["split_k"], -(-s.K // 64))
         expect += tiles * split * (2 if info["cta_pair"] == 2 else 1)   # a pair unit counts on both CTAs
     assert units == expect
 
