@@ -348,16 +348,19 @@ __device__ __forceinline__ void reduce_slice(const CView& w, const float4* tile_
 // or 64 bf16 columns) every thread writes its row into a staging buffer with
 // the 128-byte swizzle (so a warp's writes hit distinct banks), then one
 // thread issues the tensor store; two 16 KB buffers alternate, and a buffer
-// is reused only after the store two chunks back has read it.  The store
-// clips rows and columns outside C.
-template <int MMA_N, bool OUT_BF16>
+// is reused only after the store two chunks back has read it.  WIDE: the
+// chunks go to consecutive 16 KB buffers from `staging` on (MMA_N * 512 bytes
+// for fp32, half that for bf16), none reused, so no chunk waits for an
+// earlier store — for a CTA's last tile, staged in its idle operand ring.
+// The store clips rows and columns outside C.
+template <int MMA_N, bool OUT_BF16, bool WIDE = false>
 __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t staging, uint32_t& stg, uint32_t taddr,
                                                int r, int et, int m0, int n0, int b) {
   constexpr int CHUNK = OUT_BF16 ? 64 : 32;
 #pragma unroll 1
   for (int c0 = 0; c0 < MMA_N; c0 += CHUNK) {
-    const uint32_t buf = staging + (stg & 1u) * 16384u;
-    if (et == 0) ptx::bulk_wait_group_read<1>();
+    const uint32_t buf = WIDE ? staging + uint32_t(c0 / CHUNK) * 16384u : staging + (stg & 1u) * 16384u;
+    if (!WIDE && et == 0) ptx::bulk_wait_group_read<1>();
     ptx::named_bar_sync(1, 128);
     const uint32_t row = buf + uint32_t(r) * 128u;
     const uint32_t sw = uint32_t(r & 7);
@@ -1088,7 +1091,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       }
     }
     // tensor stores must have read the staging buffers before the CTA leaves
-    if (EPI_TMA && et == 0) ptx::bulk_wait_group<0>();
+    // (their writes to C complete with the grid)
+    if (EPI_TMA && et == 0) ptx::bulk_wait_group_read<0>();
   }
 
   __syncthreads();

@@ -320,7 +320,15 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
           if (et == 0) w.ws_cnt[half] = 0u;     // leave the counter zeroed for the next run
         }
       } else if (w.c_tma) {
-        store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
+        if (u + n_pairs >= p.total_units) {
+          // this CTA's last tile: every MMA has completed (the accumulator is
+          // ready) and no load is left, so the operand ring is idle and
+          // stages the whole tile (128 KB fp32 / 64 KB bf16 of its 192 KB)
+          static_assert(STAGES * STAGE_BYTES >= 256 * 512, "the ring holds a whole tile half");
+          store_tile_tma<256, OUT_BF16, true>(&p.tmap_c[c.g], tiles_base, stg, taddr, r, et, m0, n0, c.b);
+        } else {
+          store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
+        }
       } else {
 #pragma unroll 1
         for (int c0 = 0; c0 < 256; c0 += 32) {
@@ -346,7 +354,10 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
         acc_phase ^= 1;
       }
     }
-    if (et == 0) ptx::bulk_wait_group<0>();
+    // the tensor stores must have read their shared-memory sources before
+    // the CTA leaves; their writes to C complete with the grid, which is
+    // what a dependent launch's griddepcontrol.wait waits for
+    if (et == 0) ptx::bulk_wait_group_read<0>();
   }
 
   __syncthreads();
