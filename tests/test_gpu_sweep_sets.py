@@ -1,0 +1,54 @@
+"""All 64 randomized sets as the report runs them, checked by the sampling
+rule for the sweep: every GEMM of at most 2 GFLOP against the fp64 oracle
+element by element, larger GEMMs on 256 seeded rows (the first and last row
+included).
+
+Each set is planned by the dynamic logic (GOLDY_PLAN_AUTO, fused waves) and
+run the way bench.py's report runs it: a prepared run per input copy (two
+copies here), replayed back to back with `inputs_ready`, so a launch's loads
+and MMAs may overlap the previous kernel's tail.  The sets cover plans of a
+single launch, of up to five launches on one stream, and of more launches
+forked onto CD streams; tensor-bound and memory-bound sets; and the two sets
+whose plan loses to the sequential run.  Both copies hold the same inputs, so
+their outputs must also be byte-identical."""
+import numpy as np
+import pytest
+import torch
+
+import bench
+from paper_2409_02227_gb300 import goldy as G
+from paper_2409_02227_gb300 import workloads as wl
+from tests.gpu_util import check_close, check_rows
+
+pytestmark = pytest.mark.gpu
+
+FULL_CHECK_FLOPS = 2e9
+SAMPLED_ROWS = 256
+SETS = list(range(wl.SWEEP_SETS))
+
+
+@pytest.mark.parametrize("j", SETS)
+def test_sweep_set_as_reported(cuda_ok, j):
+    st = wl.make_sweep_set(j)
+    lut = G.goldy_lut_load(G.DEFAULT_LUT)
+    descs, sched, plan, single = bench.plan_set(G, st, lut, G.GOLDY_PLAN_FUSED)
+    r = bench.SetRunner(st, sched, 2)
+    for _, _, C in r.copies:
+        for c in C:
+            c.fill_(float("nan"))
+    torch.cuda.synchronize()
+    r.timed(6)
+    torch.cuda.synchronize()
+    assert G.goldy_device_error(clear=True) == 0
+    first = [c.cpu() for c in r.copies[0][2]]
+    second = [c.cpu() for c in r.copies[1][2]]
+    rng = np.random.default_rng(9000 + j)
+    for i, s in enumerate(st.specs):
+        label = f"sweep {j} gemm {i} {s.M}x{s.N}x{s.K}"
+        if s.flops <= FULL_CHECK_FLOPS:
+            check_close(first[i], st.a[i], st.b[i], label)
+        else:
+            rows = np.unique(np.concatenate([[0, s.M - 1], rng.choice(s.M, size=min(SAMPLED_ROWS - 2, s.M),
+                                                                      replace=False)]))
+            check_rows(first[i], st.a[i], st.b[i], rows, label + " (sampled rows)")
+        assert torch.equal(second[i].view(torch.uint8), first[i].view(torch.uint8)), label + ": copies differ"
