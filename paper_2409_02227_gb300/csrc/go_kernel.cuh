@@ -655,8 +655,11 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // Early mode: the producer (reading A and B only, asserted not written by
   // an earlier kernel) and the MMA thread (shared and tensor memory only)
   // go ahead; the epilogue, which writes C and the workspace, still waits.
-  // A launch that hands units out from a workspace counter always waits.
-  const bool early = p.early_loads != 0 && p.dyn == nullptr && warp < 2;
+  // A launch that hands units out from a workspace counter loads its first
+  // unit (this CTA's own) early too; the producer waits before its first
+  // read of the counter, which the previous launch over the same GEMMs
+  // zeroes as it ends.
+  const bool early = p.early_loads != 0 && warp < 2;
   if (!early) ptx::griddep_wait();
   if (threadIdx.x == 64) trace_stamp(trace, kTrSetup);   // the first epilogue thread always waits
 
@@ -684,8 +687,11 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
         if (u >= p.total_units) break;
         ++taken;
         // the next unit, taken now so that the counter's latency overlaps
-        // this unit's loads
-        const int next = p.dyn ? int(gridDim.x + atomicAdd(p.dyn, 1u)) : u + int(gridDim.x);
+        // this unit's loads — except after an early start, where the counter
+        // is read once the first unit's loads are out and the previous grid
+        // is done
+        const bool defer_next = p.dyn && early && seq == 0;
+        int next = defer_next ? 0 : (p.dyn ? int(gridDim.x + atomicAdd(p.dyn, 1u)) : u + int(gridDim.x));
         if (issued == 0) trace_stamp(trace, kTrProducerGo);
         const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
         const void* ta = &p.tmap_a[c.g];
@@ -732,6 +738,11 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
             stage = 0;
             phase ^= 1;
           }
+        }
+        if (defer_next) {
+          if (!ok || stalled) break;
+          ptx::griddep_wait();
+          next = int(gridDim.x + atomicAdd(p.dyn, 1u));
         }
         u = next;
       }
