@@ -350,9 +350,10 @@ __device__ __forceinline__ void reduce_slice(const CView& w, const float4* tile_
 // thread issues the tensor store; two 16 KB buffers alternate, and a buffer
 // is reused only after the store two chunks back has read it.  WIDE: the
 // chunks go to consecutive 16 KB buffers from `staging` on (MMA_N * 512 bytes
-// for fp32, half that for bf16), none reused, so no chunk waits for an
-// earlier store — for a CTA's last tile, staged in its idle operand ring.
-// The store clips rows and columns outside C.
+// for fp32, half that for bf16), none reused, and only the staging is done
+// here (shared memory only; issue_tile_wide stores them) — for a CTA's last
+// tile, staged in its idle operand ring.  The store clips rows and columns
+// outside C.
 template <int MMA_N, bool OUT_BF16, bool WIDE = false>
 __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t staging, uint32_t& stg, uint32_t taddr,
                                                int r, int et, int m0, int n0, int b) {
@@ -396,6 +397,7 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
                           pk[4 * j + 3]);
     }
     ptx::fence_proxy_async_smem();
+    if (WIDE) continue;
     ptx::named_bar_sync(1, 128);
     if (et == 0) {
       ptx::tma_store_3d(tmap_c, buf, n0 + c0, m0, b);
@@ -403,6 +405,19 @@ __device__ __forceinline__ void store_tile_tma(const void* tmap_c, uint32_t stag
     }
     ++stg;
   }
+  if (WIDE) ptx::named_bar_sync(1, 128);   // every chunk staged and fenced
+}
+
+// The tensor stores of a tile staged by store_tile_tma<..., true> (one
+// thread issues them all, one bulk group).
+template <int MMA_N, bool OUT_BF16>
+__device__ __forceinline__ void issue_tile_wide(const void* tmap_c, uint32_t staging, int et, int m0, int n0, int b) {
+  constexpr int CHUNK = OUT_BF16 ? 64 : 32;
+  if (et != 0) return;
+#pragma unroll 1
+  for (int c0 = 0; c0 < MMA_N; c0 += CHUNK)
+    ptx::tma_store_3d(tmap_c, staging + uint32_t(c0 / CHUNK) * 16384u, n0 + c0, m0, b);
+  ptx::bulk_commit_group();
 }
 
 // Shared-memory layout of a whole fp32 partial tile for the on-chip cluster
@@ -660,8 +675,12 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   // read of the counter, which the previous launch over the same GEMMs
   // zeroes as it ends.
   const bool early = p.early_loads != 0 && warp < 2;
-  if (!early) ptx::griddep_wait();
-  if (threadIdx.x == 64) trace_stamp(trace, kTrSetup);   // the first epilogue thread always waits
+  // In early mode the epilogue waits where it first writes global memory
+  // (below): a CTA's last tile is read out of tensor memory into the idle
+  // operand ring before that wait, so only its stores are left after it.
+  const bool epi_defer = p.early_loads != 0 && warp >= 2;
+  if (!early && !epi_defer) ptx::griddep_wait();
+  if (threadIdx.x == 64 && !epi_defer) trace_stamp(trace, kTrSetup);   // the first epilogue thread waits
 
   if (warp == 0) {
     if (lane == 0) {
@@ -836,6 +855,13 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     uint32_t red_it = 0;                    // cluster reductions done by this CTA
     uint32_t stg = 0;                       // staging buffers used (TMA-store epilogue)
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
+    bool waited = !epi_defer;               // past the wait for the previous grid
+    auto wait_prev = [&]() {
+      if (waited) return;
+      ptx::griddep_wait();
+      waited = true;
+      if (et == 0) trace_stamp(trace, kTrSetup);
+    };
     for (int seq = 0;; ++seq) {
       const int slot = seq % kUnitRing;
       int u = int(blockIdx.x) + seq * int(gridDim.x);     // static round-robin
@@ -869,7 +895,20 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const int m0 = c.tm * TILE_M;
       const int n0 = c.tn * TILE_N;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);
-      if (EPI_TMA && w.split == 1 && w.c_tma) {
+      // this CTA's last tile with nothing but tensor stores: the operand
+      // ring is idle (every MMA done, no load left) and stages all of it
+      const bool wide = EPI_TMA && w.split == 1 && w.c_tma && p.dyn == nullptr &&
+                        u + int(gridDim.x) >= p.total_units;
+      static_assert(!EPI_TMA || STAGES * STAGE_BYTES >= MMA_N * 512, "the ring holds a whole tile");
+      if (wide) {
+        store_tile_tma<MMA_N, OUT_BF16, true>(&p.tmap_c[c.g], tiles_base, stg, taddr, r, et, m0, n0, c.b);
+        wait_prev();
+        issue_tile_wide<MMA_N, OUT_BF16>(&p.tmap_c[c.g], tiles_base, et, m0, n0, c.b);
+      } else {
+        wait_prev();
+      }
+      if (wide) {
+      } else if (EPI_TMA && w.split == 1 && w.c_tma) {
         store_tile_tma<MMA_N, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
       } else if (w.split == 1) {
 #pragma unroll 1

@@ -119,8 +119,11 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
   // global memory only after the previous grid is done; in early mode the
   // load and MMA roles go ahead (see go_gemm_kernel) and the epilogue waits
   const bool early = p.early_loads != 0 && warp < 2;
-  if (!early) ptx::griddep_wait();
-  if (threadIdx.x == 64) trace_stamp(trace, kTrSetup);   // the first epilogue thread always waits
+  // in early mode the epilogue waits where it first writes global memory
+  // (below); a CTA's last tile is staged in the idle ring before that wait
+  const bool epi_defer = p.early_loads != 0 && warp >= 2;
+  if (!early && !epi_defer) ptx::griddep_wait();
+  if (threadIdx.x == 64 && !epi_defer) trace_stamp(trace, kTrSetup);   // the first epilogue thread waits
 
   if (warp == 0) {
     if (lane == 0) {
@@ -241,6 +244,13 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
     uint32_t acc_phase = 0;
     uint32_t stg = 0;
     const uint32_t staging = tiles_base + STAGES * STAGE_BYTES;
+    bool waited = !epi_defer;               // past the wait for the previous grid
+    auto wait_prev = [&]() {
+      if (waited) return;
+      ptx::griddep_wait();
+      waited = true;
+      if (et == 0) trace_stamp(trace, kTrSetup);
+    };
     for (int u = pair; u < p.total_units; u += n_pairs) {
       const UnitCoord c = decode_unit_tab(utab, n_gemms, u);
       const GemmWork w = p.g[c.g];                 // read while the accumulator is computed
@@ -257,7 +267,21 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
       const int m0 = c.tm * 256 + int(rank) * 128;
       const int n0 = c.tn * 256;
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * 256);
-      if (w.split > 1) {
+      // this CTA's last tile: every MMA has completed (the accumulator is
+      // ready) and no load is left, so the operand ring is idle and stages
+      // the whole tile (128 KB fp32 / 64 KB bf16 of its 192 KB) before the
+      // wait; only the stores follow it
+      const bool wide = w.split == 1 && w.c_tma && u + n_pairs >= p.total_units;
+      static_assert(STAGES * STAGE_BYTES >= 256 * 512, "the ring holds a whole tile half");
+      if (wide) {
+        store_tile_tma<256, OUT_BF16, true>(&p.tmap_c[c.g], tiles_base, stg, taddr, r, et, m0, n0, c.b);
+        wait_prev();
+        issue_tile_wide<256, OUT_BF16>(&p.tmap_c[c.g], tiles_base, et, m0, n0, c.b);
+      } else {
+        wait_prev();
+      }
+      if (wide) {
+      } else if (w.split > 1) {
         // ---- split-K: this CTA publishes its fp32 partial (its 128 rows of
         // the 256 x 256 tile, layout [chunk][float4][row]) to the workspace
         // and counts itself in; the last of the S splits to arrive for this
@@ -320,15 +344,7 @@ __global__ void __launch_bounds__(192, 1) go_gemm_pair_kernel(const __grid_const
           if (et == 0) w.ws_cnt[half] = 0u;     // leave the counter zeroed for the next run
         }
       } else if (w.c_tma) {
-        if (u + n_pairs >= p.total_units) {
-          // this CTA's last tile: every MMA has completed (the accumulator is
-          // ready) and no load is left, so the operand ring is idle and
-          // stages the whole tile (128 KB fp32 / 64 KB bf16 of its 192 KB)
-          static_assert(STAGES * STAGE_BYTES >= 256 * 512, "the ring holds a whole tile half");
-          store_tile_tma<256, OUT_BF16, true>(&p.tmap_c[c.g], tiles_base, stg, taddr, r, et, m0, n0, c.b);
-        } else {
-          store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
-        }
+        store_tile_tma<256, OUT_BF16>(&p.tmap_c[c.g], staging, stg, taddr, r, et, m0, n0, c.b);
       } else {
 #pragma unroll 1
         for (int c0 = 0; c0 < 256; c0 += 32) {
