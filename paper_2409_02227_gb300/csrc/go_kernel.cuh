@@ -900,11 +900,14 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const bool wide = EPI_TMA && w.split == 1 && w.c_tma && p.dyn == nullptr &&
                         u + int(gridDim.x) >= p.total_units;
       static_assert(!EPI_TMA || STAGES * STAGE_BYTES >= MMA_N * 512, "the ring holds a whole tile");
+      // the cluster reductions on chip exchange partials through shared
+      // memory only and wait just before their stores
+      const bool onchip = kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x);
       if (wide) {
         store_tile_tma<MMA_N, OUT_BF16, true>(&p.tmap_c[c.g], tiles_base, stg, taddr, r, et, m0, n0, c.b);
         wait_prev();
         issue_tile_wide<MMA_N, OUT_BF16>(&p.tmap_c[c.g], tiles_base, et, m0, n0, c.b);
-      } else {
+      } else if (!(w.split > 1 && (push_on || onchip))) {
         wait_prev();
       }
       if (wide) {
@@ -975,6 +978,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           break;
         }
         if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
+        wait_prev();
         const uint32_t own_slot = tiles_base + uint32_t(c.s) * slot_bytes;
         switch (S) {
           case 2: reduce_slice_pushed<MMA_N, 2, SWAP, OUT_BF16>(cv, own_slot, recv_slots, c.s, m0, n0, et); break;
@@ -982,7 +986,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           case 8: reduce_slice_pushed<MMA_N, 8, SWAP, OUT_BF16>(cv, own_slot, recv_slots, c.s, m0, n0, et); break;
           default: break;
         }
-      } else if (kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x)) {
+      } else if (onchip) {
         // ---- cluster split-K on chip: one unit per CTA, so the ring's shared
         // memory is free once the accumulator is complete.  Publish the fp32
         // partial there, signal every peer, wait for all S partials, reduce
@@ -1019,6 +1023,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
           break;
         }
         if (first_unit && et == 0) trace_stamp(trace, kTrArrived);
+        wait_prev();
         switch (w.split) {
           case 2: reduce_slice_dsmem<MMA_N, 2, SWAP, OUT_BF16>(cv, part_smem, c.s, m0, n0, et); break;
           case 4: reduce_slice_dsmem<MMA_N, 4, SWAP, OUT_BF16>(cv, part_smem, c.s, m0, n0, et); break;
