@@ -543,6 +543,8 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
   constexpr int TILE_M = SWAP ? MMA_N : 128;         // C rows per tile
   constexpr int TILE_N = SWAP ? 128 : MMA_N;         // C columns per tile
   constexpr int B_BOXES = TILE_N / 64;               // 64-column TMA boxes of B per stage
+  // a CTA's last tile can be staged whole in the operand ring (see the epilogue)
+  constexpr bool kWideFits = !SWAP && STAGES * STAGE_BYTES >= 128 * MMA_N * (OUT_BF16 ? 2 : 4);
   constexpr uint32_t TMEM_COLS = TmemCols<MMA_N, ACC>::value;
   // !SWAP: MMA-A = A tile (K-major), MMA-B = B tile (N-major)
   //  SWAP: MMA-A = B tile (N-major), MMA-B = A tile (K-major)
@@ -897,9 +899,11 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
       const uint32_t taddr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(acc * MMA_N);
       // this CTA's last tile with nothing but tensor stores: the operand
       // ring is idle (every MMA done, no load left) and stages all of it
-      const bool wide = EPI_TMA && w.split == 1 && w.c_tma && p.dyn == nullptr &&
+      // (two-per-SM kinds too, where their ring holds the tile: they keep no
+      // staging buffers and store their other tiles directly)
+      static_assert(!EPI_TMA || kWideFits, "the ring holds a whole tile");
+      const bool wide = kWideFits && w.split == 1 && w.c_tma && p.dyn == nullptr &&
                         u + int(gridDim.x) >= p.total_units;
-      static_assert(!EPI_TMA || STAGES * STAGE_BYTES >= MMA_N * 512, "the ring holds a whole tile");
       // the cluster reductions on chip exchange partials through shared
       // memory only and wait just before their stores
       const bool onchip = kPartFitsRing && p.cluster > 0 && p.total_units == int(gridDim.x);
@@ -1147,7 +1151,7 @@ __global__ void __launch_bounds__(192, MIN_CTAS) go_gemm_kernel(const __grid_con
     }
     // tensor stores must have read the staging buffers before the CTA leaves
     // (their writes to C complete with the grid)
-    if (EPI_TMA && et == 0) ptx::bulk_wait_group_read<0>();
+    if ((EPI_TMA || kWideFits) && et == 0) ptx::bulk_wait_group_read<0>();
   }
 
   __syncthreads();

@@ -412,9 +412,12 @@ goldy_status fill_slot(LaunchParams<MAXG>& p, int j, const GemmPlan& gp, const v
   // C through TMA stores: kinds that keep staging buffers, 16-byte aligned C
   // and rows; the epilogue writes 128-byte rows (32 fp32 / 64 bf16 columns)
   const size_t es = g.c_dtype == GOLDY_BF16 ? 2 : 4;
+  // (kinds with a whole SM store every tile this way; the two-per-SM kinds,
+  // which keep no staging buffers, only a CTA's last tile, staged in its
+  // idle operand ring)
   w.c_tma = 0;
   const uint64_t sc = uint64_t(w.c_bstride) * es;
-  if (epi_tma(k) && gp.split == 1 && aligned(C, 16) && (size_t(g.ldc) * es) % 16 == 0 && sc % 16 == 0) {
+  if (!k.swap_ab && gp.split == 1 && aligned(C, 16) && (size_t(g.ldc) * es) % 16 == 0 && sc % 16 == 0) {
     st = encode_3d(&p.tmap_c[j], C, uint64_t(g.N), uint64_t(g.M), uint64_t(g.batch), uint64_t(g.ldc) * es, sc,
                    uint32_t(128 / es), 128,
                    g.c_dtype == GOLDY_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
