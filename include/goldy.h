@@ -109,8 +109,8 @@ typedef struct goldy_graph goldy_graph;
  * (outside a stream capture the other streams also wait until all of its
  * CTAs have begun).  Groups are not separated by a join: the run forks once
  * and joins once, and a later group's launches take lower priorities, so they
- * fill the SMs an earlier group frees.  A fused run of at most 5 launches
- * run with goldy_run_opts.inputs_ready = 1 goes out on streams[0] alone
+ * fill the SMs an earlier group frees.  A fused run with
+ * goldy_run_opts.inputs_ready = 1 goes out on streams[0] alone
  * instead, each wave's largest launch first, every launch overlapping the
  * previous one's tail (no fork, no join).  Without FUSED every GEMM is its own
  * launch on its slot's stream and the groups run one after another.  The plan

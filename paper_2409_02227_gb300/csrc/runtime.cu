@@ -83,9 +83,6 @@ thread_local bool t_pdl = true;
 // early operand loads, the bounded-wait limit, and the test stall hook
 // (first launch of the run only).
 thread_local int32_t t_early = 0;
-// Fused runs of at most this many launches go out on one stream when the
-// caller declared its inputs ready (see run_impl).
-constexpr int kOneStreamLaunches = 5;
 thread_local uint64_t t_wait_ns = 0;
 thread_local int32_t t_stall = 0;
 // Launch priority of the next GO-Kernel launch (kNoPriority: the stream's).
@@ -983,20 +980,22 @@ static goldy_status run_impl(const goldy_schedule* s, const void* const* A, cons
     // and waits measured ~4 us on a two-GEMM set of small kernels
     if (kernels < 2 || (lead < sets.size() && !kKinds[s->gemms[sets[lead].members[0]].kind].pair)) lead = sets.size();
   }
-  // Fused runs of few launches with inputs_ready go out on streams[0] alone,
-  // largest launch of each wave first: each launch's loads and MMAs start in
-  // the previous one's tail (programmatic dependent launch), with no fork or
-  // join, and consecutive runs overlap the same way.  Runs of more launches
-  // keep the CD streams, where a later wave or group's launches need not
-  // wait for the earlier ones to complete.  Measured over the 64 randomized
-  // sets, back to back (launches per run <= L on one stream): roofline
-  // fraction geomean 0.381 (L = 0), 0.400 (2), 0.408 (3), 0.414 (4), 0.416
-  // (5), 0.415 (6), 0.410 (all); the sets of two or three launches gained up
-  // to 2x.  Without inputs_ready a launch would wait for the previous one to
+  // Fused runs with inputs_ready go out on streams[0] alone, largest launch
+  // of each wave first: each launch's loads and MMAs start in the previous
+  // one's tail (programmatic dependent launch), with no fork or join, and
+  // consecutive runs overlap the same way; each launch's epilogue waits for
+  // the previous kernel only where it first writes global memory.  Measured
+  // over the 64 randomized sets, back to back: with runs of at most 5
+  // launches on one stream and the rest on the CD streams, roofline
+  // fraction geomean 0.443 (tensor-bound 0.556); with every run on one
+  // stream 0.446 (0.561), runs of 6-9 launches up to 13% faster, two of them
+  // 5-8% slower.  (Before the epilogues waited only at their first global
+  // write, runs of more than 5 launches measured 4-6% slower on one stream.)
+  // Without inputs_ready a launch would wait for the previous one to
   // complete, so those runs keep the streams.
   int n_launches = 0;
   for (const LaunchSet& ls : sets) n_launches += ls.degenerate ? 0 : 1;
-  const bool one_stream = fused && t_early && n_launches >= 2 && n_launches <= kOneStreamLaunches;
+  const bool one_stream = fused && t_early && n_launches >= 2;
   if (one_stream) lead = sets.size();
   std::vector<size_t> order;
   order.reserve(sets.size());

@@ -386,9 +386,10 @@ def test_one_kind_per_wave_plans_match_oracle(cuda_ok, j):
 @pytest.mark.parametrize("j", [30, 48, 16])
 def test_few_launch_runs_on_one_stream_match(cuda_ok, j):
     # randomized sets whose fused plan has 2 to 5 launches: with inputs_ready
-    # they go out on streams[0] alone (each wave's largest first); replayed
-    # back to back as prepared runs they give the same bytes as the forked
-    # multi-stream run without the option, and the oracle's values
+    # they (like every fused run) go out on streams[0] alone, each wave's
+    # largest first; replayed back to back as prepared runs they give the
+    # same bytes as the forked multi-stream run without the option, and the
+    # oracle's values
     st = wl.make_sweep_set(j)
     descs = [G.desc(s.M, s.N, s.K, s.out_dtype) for s in st.specs]
     sched = G.goldy_plan(descs, G.goldy_lut_load(G.DEFAULT_LUT), G.GOLDY_PLAN_AUTO | G.GOLDY_PLAN_FUSED)

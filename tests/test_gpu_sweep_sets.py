@@ -6,10 +6,9 @@ included).
 Each set is planned by the dynamic logic (GOLDY_PLAN_AUTO, fused waves) and
 run the way bench.py's report runs it: a prepared run per input copy (two
 copies here), replayed back to back with `inputs_ready`, so a launch's loads
-and MMAs may overlap the previous kernel's tail.  The sets cover plans of a
-single launch, of up to five launches on one stream, and of more launches
-forked onto CD streams; tensor-bound and memory-bound sets; and the two sets
-whose plan loses to the sequential run.  Both copies hold the same inputs, so
+and MMAs may overlap the previous kernel's tail, and every run goes out on
+one stream.  The sets' plans range from a single launch to nine, over
+tensor-bound and memory-bound sets.  Both copies hold the same inputs, so
 their outputs must also be byte-identical."""
 import numpy as np
 import pytest
